@@ -1,0 +1,374 @@
+"""Throughput of the batched multi-tier scheduler simulation on GB300.
+
+A step is one complete simulation of the benchmark workload -- 1,024
+independent replicas, each a 16-instance x 2,048-block cluster with K = 4
+enterprise-mix tiers and 20,000 requests (Poisson at 0.85 of capacity) -- from
+t = 0 until every request has finished: state reset plus one persistent
+simulation kernel, inputs resident in HBM.  `value` is simulated
+replica-steps per second (a replica-step = one distinct event time processed in
+one replica), summed over GPUs.  `e2e` repeats the measurement through the C
+ABI with the trace in pinned host memory: the host-to-device copy, validation,
+simulation and the device-to-host copy of every per-request result are inside
+the timed region.
+
+Multi-GPU (torchrun, one process per GPU): each rank simulates its own
+independent copy of the workload (other seeds); there is no collective on the
+data path, only a barrier and a max/sum of the timings (weak scaling).
+
+--impl reference times the CPU oracle (the plain single-threaded reference
+simulator, one replica per host thread) on a bounded sample of the same
+workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+if HERE not in sys.path:
+    sys.path.insert(0, HERE)
+
+import numpy as np  # noqa: E402
+
+WORKLOAD_ID = 1
+WORKLOAD_NAME = ("1,024 replicas x 16 instances x 2,048 KV blocks (16 tokens/block, batch 64), K=4 enterprise tiers "
+                 "(.05/.15/.30/.50), 20,000 requests/replica, Poisson at 0.85 load, H_k = 512 >> k, "
+                 "64 migration blocks/iteration, 50 ms / theta 0.3 rebalancing")
+METRIC = "simulated replica-steps/sec (1 GB300) and achieved HBM GB/s fraction of peak"
+UNIT = "replica-steps/s"
+# Algorithmic bytes (what the method must move through HBM at minimum):
+BYTES_PER_REQUEST = 9 + 16       # read the trace record, write the result record
+BYTES_PER_MEMBER_ITERATION = 8   # read + write a running request's 2-byte token and 2-byte block counters
+BYTES_PER_LOG_RECORD = 16        # one migration-log record
+KERNELS_PER_STEP = 3             # k_init_state, k_init_requests, k_run
+
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", str(rank)))
+    return ws, rank, local
+
+
+def aggregate(local_seconds: float, local_units: float, local_events: float):
+    """Max of the timings and sum of the work over ranks (identity at N = 1)."""
+    import torch
+    import torch.distributed as dist
+
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return local_seconds, local_units, local_events
+    dev = torch.device("cuda") if dist.get_backend() == "nccl" else torch.device("cpu")
+    t = torch.tensor([local_seconds], dtype=torch.float64, device=dev)
+    u = torch.tensor([local_units, local_events], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.all_reduce(u, op=dist.ReduceOp.SUM)
+    return float(t.item()), float(u[0].item()), float(u[1].item())
+
+
+def barrier():
+    import torch.distributed as dist
+
+    if dist.is_available() and dist.is_initialized():
+        dist.barrier()
+
+
+def measured_peak_hbm():
+    path = os.path.join(HERE, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def kernel_traffic(per_launch_units: float):
+    """DRAM bytes per k_run launch from the committed ncu summary, scaled to
+    this launch, or None if the kernel source changed since the capture."""
+    path = os.path.join(HERE, "profiles", "k_run_workload1_traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)
+        import hashlib
+
+        src = os.path.join(HERE, "paper_2608_16336_gb300", "csrc", "mtsim.cu")
+        if hashlib.sha256(open(src, "rb").read()).hexdigest() != rec["mtsim_cu_sha256"]:
+            return None
+        return float(rec["dram_bytes_per_unit"]) * per_launch_units
+    except Exception:
+        return None
+
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons during the timed region."""
+
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = os.path.join(HERE, "gpurun_out", "clocks_bench_%d.csv" % gpu_index)
+
+    def start(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + self.QUERY,
+                                          "--format=csv,noheader,nounits", "-lms", "200"], stdout=self.f,
+                                         stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if not self.proc:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.f.close()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def bench_gpu(args):
+    import torch
+
+    ws, rank, local = dist_env()
+    if ws > 1:
+        import torch.distributed as dist
+
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    else:
+        torch.cuda.set_device(0)
+    from paper_2608_16336_gb300 import mtsim, workloads
+
+    reps = range(args.replicas) if args.replicas else None
+    w = workloads.config(WORKLOAD_ID, replicas=reps, requests=args.requests, seed_block=rank)
+    stream = torch.cuda.current_stream()
+    sim = mtsim.Simulator(w, event_log_capacity=args.log_capacity, stream=stream)
+    sim.load(on_device=True)
+    R, Q = w.num_replicas, w.total_requests
+
+    def step():
+        mtsim.sim_reset(sim.handle)
+        mtsim.sim_run(sim.handle, 1 << 62, False)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    # per-launch duration of the simulation kernel, on its own stream
+    k_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    clocks = ClockSampler(local)
+    clocks.start()
+    barrier()
+    torch.cuda.synchronize()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for i in range(args.steps):
+        mtsim.sim_reset(sim.handle)
+        k_ev[i][0].record(stream)
+        mtsim.sim_run(sim.handle, 1 << 62, False)
+        k_ev[i][1].record(stream)
+    t1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    clk = clocks.stop()
+    dev_s = t0.elapsed_time(t1) / 1e3
+    k_s = sum(a.elapsed_time(b) for a, b in k_ev) / 1e3 / args.steps
+
+    res, st, _ = sim.metrics()
+    assert (st["status"] == mtsim.SIM_REPLICA_DONE).all(), "a replica did not finish"
+    steps_per_run = float(st["steps"].sum())
+    events_per_run = float(st["events"].sum())
+    member_iters = float(st["member_iterations"].sum())
+    log_recs = float(np.minimum(st["log_events"], args.log_capacity).sum())
+    alg_bytes = Q * BYTES_PER_REQUEST + member_iters * BYTES_PER_MEMBER_ITERATION + log_recs * BYTES_PER_LOG_RECORD
+
+    # end to end through the C ABI with pinned host buffers
+    pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
+    h_arr, h_p, h_o, h_t = (pin(w.arrival_us.view(np.int32)), pin(w.prompt_len.view(np.int16)),
+                            pin(w.output_len.view(np.int16)), pin(w.tier))
+    h_res = torch.empty(Q * 16, dtype=torch.uint8).pin_memory()
+    h_st = torch.empty(R * 64, dtype=torch.uint8).pin_memory()
+    off = np.ascontiguousarray(w.offsets, np.int64)
+
+    def e2e_step():
+        mtsim.sim_load_trace(sim.handle, off.ctypes.data, h_arr.data_ptr(), h_p.data_ptr(), h_o.data_ptr(),
+                             h_t.data_ptr(), 0)
+        mtsim.sim_run(sim.handle, 1 << 62, False)
+        mtsim.sim_metrics(sim.handle, h_res.data_ptr(), h_st.data_ptr(), None, 0)
+
+    e2e_step()
+    barrier()
+    torch.cuda.synchronize()
+    e0 = time.perf_counter()
+    for _ in range(args.e2e_steps):
+        e2e_step()
+    torch.cuda.synchronize()
+    barrier()
+    e2e_s = (time.perf_counter() - e0) / args.e2e_steps
+    h2d = int(off.nbytes + Q * 9)
+    d2h = int(Q * 16 + R * 64)
+    sim.close()
+
+    tot_s, tot_units, tot_events = aggregate(dev_s, steps_per_run * args.steps, events_per_run * args.steps)
+    e2e_max, e2e_units, _ = aggregate(e2e_s, steps_per_run, events_per_run)
+    peak, peak_kind = measured_peak_hbm()
+    achieved = alg_bytes / k_s / 1e9
+    line = {
+        "metric": METRIC,
+        "value": tot_units / tot_s,
+        "unit": UNIT,
+        "n_gpus": ws,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": tot_s / args.steps * 1e3,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "int32",
+        "data": "synthetic (seeded traces shaped like the paper's workloads; no dataset)",
+        "config": {
+            "workload": WORKLOAD_NAME if not (args.replicas or args.requests) else
+            "REDUCED profiling case of: " + WORKLOAD_NAME,
+            "replicas_per_gpu": R,
+            "requests_per_gpu": Q,
+            "replica_steps_per_gpu_step": int(steps_per_run),
+            "parallelism": "replicas sharded across GPUs, no collective on the data path",
+            "l2": "inputs larger than L2: trace %.0f MB + per-request state %.0f MB resident" % (
+                Q * 9 / 1e6, Q * 26 / 1e6),
+        },
+        "request_events_per_s": tot_events / tot_s,
+        "e2e": {"value": e2e_units / e2e_max, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": KERNELS_PER_STEP * args.steps,
+        "roofline": {
+            "bound": "hbm",
+            "achieved": achieved,
+            "peak": peak,
+            "peak_kind": peak_kind,
+            "unit": "GB/s",
+            "frac": achieved / peak,
+            "traffic": kernel_traffic(Q),
+            "kernel": "k_run",
+            "kernel_ms": k_s * 1e3,
+            "algorithmic_bytes_per_launch": alg_bytes,
+        },
+        "clocks": clk,
+    }
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(w, args.cpu_replicas)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if ws > 1:
+        import torch.distributed as dist
+
+        dist.destroy_process_group()
+
+
+def cpu_baseline(w, nrep: int) -> dict:
+    """The oracle, as it stands, on the first `nrep` replicas of the same workload,
+    one replica per host thread on all host cores."""
+    from oracle import oracle
+
+    cores = os.cpu_count() or 1
+    reps = list(range(min(nrep, w.num_replicas)))
+    r = oracle.timed_sample(w, reps, cores)
+    return {"value": r["steps"] / r["seconds"], "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": "first %d of %d replicas, full 20,000 requests each (%d replica-steps, %.1f s wall)" % (
+                len(reps), w.num_replicas, r["steps"], r["seconds"]),
+            "request_events_per_s": r["events"] / r["seconds"]}
+
+
+def bench_reference(args):
+    ws, rank, _ = dist_env()
+    if rank != 0:
+        return
+    from oracle import oracle
+    from paper_2608_16336_gb300 import workloads
+
+    w = workloads.config(WORKLOAD_ID)
+    cores = os.cpu_count() or 1
+    reps = list(range(min(args.cpu_replicas_per_step, w.num_replicas)))
+    for _ in range(args.warmup):
+        oracle.timed_sample(w, reps[: max(1, cores)], cores)
+    tot_s, tot_steps, tot_events = 0.0, 0, 0
+    for i in range(args.steps):
+        r = oracle.timed_sample(w, reps, cores)
+        tot_s += r["seconds"]
+        tot_steps += r["steps"]
+        tot_events += r["events"]
+    value = tot_steps / tot_s
+    line = {
+        "impl": "reference",
+        "metric": METRIC,
+        "value": value,
+        "unit": UNIT,
+        "n_gpus": ws,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": tot_s / args.steps * 1e3,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "int64",
+        "data": "synthetic (seeded traces shaped like the paper's workloads; no dataset)",
+        "config": {"workload": WORKLOAD_NAME,
+                   "sample_per_step": "first %d of 1,024 replicas, full requests" % len(reps)},
+        "request_events_per_s": tot_events / tot_s,
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": "first %d of 1,024 replicas per step" % len(reps)},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="native", choices=["native", "reference"])
+    ap.add_argument("--e2e-steps", type=int, default=2)
+    ap.add_argument("--log-capacity", type=int, default=4096)
+    ap.add_argument("--cpu-replicas", type=int, default=256)
+    ap.add_argument("--cpu-replicas-per-step", type=int, default=64)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--replicas", type=int, default=0, help="profiling only: first N replicas of the workload")
+    ap.add_argument("--requests", type=int, default=None, help="profiling only: requests per replica")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        raise SystemExit("at least 3 warm-up steps are required")
+    if args.impl == "reference":
+        bench_reference(args)
+    else:
+        bench_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

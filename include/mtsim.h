@@ -1,0 +1,231 @@
+/*
+ * mtsim.h -- C ABI of libmtsim, a batched GPU simulation of the multi-tier
+ * Llumnix-style LLM-serving scheduler of "Beyond Binary Priorities:
+ * Multi-Tier SLA Scheduling for LLM Serving" (Sec. 3).
+ *
+ * One simulation object holds R independent replicas.  A replica is a
+ * serving cluster of N instances ("Llumlets", Sec. 3.1) with M KV-cache blocks
+ * of T tokens each and a maximum running batch of Bmax requests, fed by its
+ * own request trace.  Each simulation step of a replica processes every event
+ * at the replica's next event time t, in this order:
+ *   1. iteration ends at instances whose batch finishes at t (token
+ *      accounting, request completion, one copy stage of an outbound
+ *      migration, Sec. 3.5 Fig. 4);
+ *   2. dispatch of the requests arriving at t, tier 0 first and FCFS within a
+ *      tier, each to the instance of highest freeness F (Sec. 3.4), where
+ *      F = (M - sum_r V(r)) / B (Sec. 3.2 Eq. 1-2) and the virtual usage
+ *      includes the per-tier headroom H_k of every tier present, charged once
+ *      per tier (Sec. 3.3 Eq. 3-4);
+ *   3. at every migration interval, pairing of low- and high-freeness
+ *      instances while max F - min F >= theta (Sec. 3.5);
+ *   4. batch formation at idle instances (continuous batching with
+ *      priority-ordered queues, KV growth and preemption, Sec. 2.2, 3.1) under
+ *      the integer iteration-time model base + a*prefill_tokens + b*decodes.
+ * All quantities are integers (blocks, tokens, microseconds); freeness is
+ * compared exactly.  Results are deterministic and independent of how the
+ * replicas are batched or how a run is split into sim_run calls.
+ *
+ * Conventions for every entry point:
+ *  - Return value: SIM_OK (0) or a negative SIM_ERR_* code; sim_last_error()
+ *    then describes the failure.  A failed call leaves the object usable
+ *    unless the code is SIM_ERR_CUDA.
+ *  - Pointers named "host" are host memory; pointers documented as
+ *    "host or device" follow the call's on_device flag (0 = host, 1 = device
+ *    memory of the simulation's GPU).  Input buffers are copied; the caller
+ *    keeps ownership of every buffer it passes.  The sim_t object owns all of
+ *    its device memory.
+ *  - Work is queued on the CUDA stream given to sim_create.  Calls that return
+ *    data to the host (sim_load_trace's validation, sim_run with a non-NULL
+ *    num_unfinished, sim_metrics) synchronise that stream; nothing else does.
+ *  - An object must not be used from two host threads at once.
+ */
+#ifndef MTSIM_H
+#define MTSIM_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ------------------------------------------------------------- limits --- */
+#define SIM_MAX_TIERS 16        /* K <= 16 priority tiers, tier 0 highest (Sec. 4.2) */
+#define SIM_MAX_INSTANCES 256   /* N */
+#define SIM_MAX_BATCH 64        /* Bmax */
+#define SIM_MAX_BLOCKS 65535    /* M */
+
+/* --------------------------------------------------------- return codes --- */
+#define SIM_OK 0
+#define SIM_ERR_ARG (-1)        /* invalid argument or limit exceeded */
+#define SIM_ERR_TRACE (-2)      /* malformed trace (see sim_load_trace) */
+#define SIM_ERR_STATE (-3)      /* call out of order (e.g. sim_run before sim_load_trace) */
+#define SIM_ERR_OOM (-4)        /* device allocation failed */
+#define SIM_ERR_OVERFLOW (-5)   /* a time or counter would exceed its 32-bit field */
+#define SIM_ERR_CUDA (-7)       /* CUDA runtime error; the object should be destroyed */
+#define SIM_ERR_INTERNAL (-8)   /* a device-side consistency check failed */
+#define SIM_ERR_DEADLOCK (-10)  /* no event left while requests are unfinished */
+
+/* Per-replica status (sim_replica_stats_t.status). */
+#define SIM_REPLICA_DONE 0      /* every request of the replica has finished */
+#define SIM_REPLICA_RUNNING 1   /* stopped by the step limit; sim_run resumes it */
+/* negative values: SIM_ERR_OVERFLOW, SIM_ERR_INTERNAL, SIM_ERR_DEADLOCK */
+
+#define SIM_POLICY_LLUMNIX_MT 0 /* multi-tier Llumnix global scheduler (Sec. 3) */
+
+/* Migration log record kinds (Sec. 3.5). */
+#define SIM_EV_QUEUED 0  /* a queued request moved to the destination at once (0 blocks) */
+#define SIM_EV_START 1   /* staged copy of a running request began (blocks = its KV size) */
+#define SIM_EV_COMMIT 2  /* the request committed to the destination (blocks = its KV size) */
+#define SIM_EV_ABORT 3   /* staged copy abandoned (blocks = blocks copied so far) */
+
+#define SIM_NONE32 0xFFFFFFFFu  /* "not set" for 32-bit times */
+#define SIM_NONE16 0xFFFFu      /* "not set" for 16-bit instance ids */
+
+/* ---------------------------------------------------------------- types --- */
+typedef struct sim sim_t; /* opaque, owned by the library */
+
+typedef struct {
+    int32_t num_replicas;        /* R >= 1 */
+    int32_t num_instances;       /* N in [1, SIM_MAX_INSTANCES] */
+    int32_t blocks_per_instance; /* M in [1, SIM_MAX_BLOCKS] KV blocks per instance */
+    int32_t tokens_per_block;    /* T in [1, 65535] */
+    int32_t max_batch;           /* Bmax in [1, SIM_MAX_BATCH] running requests per instance */
+} sim_cluster_t;
+
+/* Per-tier headroom H_k in blocks (Sec. 3.3 Eq. 3), one table per distinct
+ * tier setting; every replica names its table.  All pointers are host. */
+typedef struct {
+    int32_t num_tables;             /* >= 1 */
+    int32_t max_tiers;              /* row stride of headroom_blocks, in [1, SIM_MAX_TIERS] */
+    const int32_t *num_tiers;       /* [num_tables]: K of each table, in [1, max_tiers] */
+    const int32_t *headroom_blocks; /* [num_tables * max_tiers]: H_k >= 0 for k < K */
+    const int32_t *replica_table;   /* [num_replicas]: table index of each replica */
+} sim_tier_table_t;
+
+typedef struct {
+    int32_t policy;                     /* SIM_POLICY_LLUMNIX_MT */
+    int32_t enable_migration;           /* 0 or 1 */
+    int64_t iter_base_us;               /* iteration time = base */
+    int64_t iter_us_per_prefill_token;  /*   + a * prefill tokens in the batch */
+    int64_t iter_us_per_decode_seq;     /*   + b * decode requests in the batch; each in [0, 2^24] */
+    int32_t migrate_blocks_per_iter;    /* S: KV blocks copied per source iteration, in [1, 65535] */
+    int32_t theta_num, theta_den;       /* imbalance threshold theta = num/den (0.3 = 3/10) */
+    int32_t event_log_capacity;         /* migration-log records kept per replica, in [0, 2^24] */
+    int64_t migrate_interval_us;        /* rebalancing period, in [1, 2^31] (50 ms in Sec. 3.5) */
+} sim_policy_t;
+
+/* Per-request outcome, 16 bytes.  Times are microseconds from the replica's
+ * start; TTFT = first_token_us - arrival, E2E = finish_us - arrival.  The
+ * migration and preemption counters are kept modulo 2^16. */
+typedef struct {
+    uint16_t dispatch_instance;  /* instance chosen at arrival (SIM_NONE16 if not yet arrived) */
+    uint16_t final_instance;     /* instance it finished on (SIM_NONE16 if unfinished) */
+    uint32_t first_token_us;     /* SIM_NONE32 if no token yet */
+    uint32_t finish_us;          /* SIM_NONE32 if unfinished */
+    uint16_t n_migrations;       /* queued moves + committed running migrations */
+    uint16_t n_preemptions;
+} sim_request_result_t;
+
+typedef struct {
+    uint64_t steps;              /* distinct event times processed */
+    uint64_t iterations;         /* batches formed */
+    uint64_t member_iterations;  /* sum of batch sizes over all iterations */
+    uint64_t events;             /* arrivals + first tokens + finishes + migrations + preemptions */
+    uint32_t migrations;         /* queued moves + commits */
+    uint32_t preemptions;
+    uint32_t migration_starts;
+    uint32_t migration_aborts;
+    uint32_t log_events;         /* migration-log records produced (may exceed the capacity) */
+    uint32_t finished;           /* requests finished */
+    uint32_t last_time_us;       /* time of the last processed step */
+    int32_t status;              /* SIM_REPLICA_* or a negative SIM_ERR_* code */
+} sim_replica_stats_t;
+
+typedef struct {
+    uint32_t time_us;
+    uint32_t request;            /* index within the replica's trace */
+    uint16_t blocks;
+    uint8_t src, dst;            /* instance indices (N <= 256) */
+    uint8_t kind;                /* SIM_EV_* */
+    uint8_t pad[3];
+} sim_migration_event_t;
+
+/* Optional device allocator, e.g. a framework's caching allocator.  alloc
+ * returns a device pointer (16-byte aligned at least) or NULL; free releases
+ * one.  Both are called on the calling host thread with the simulation's
+ * stream.  NULL allocator: the library uses cudaMallocAsync / cudaFreeAsync
+ * on that stream. */
+typedef void *(*sim_alloc_fn)(void *ctx, size_t bytes, void *cuda_stream);
+typedef void (*sim_free_fn)(void *ctx, void *ptr, size_t bytes, void *cuda_stream);
+typedef struct {
+    void *ctx;
+    sim_alloc_fn alloc;
+    sim_free_fn free;
+} sim_allocator_t;
+
+/* ---------------------------------------------------------- entry points --- */
+
+/* Creates a simulation of cluster->num_replicas replicas on the current CUDA
+ * device.  The cluster, tier tables and policy are validated (limits above;
+ * additionally M + sum_k H_k must stay below 2^19 for every table) and
+ * copied.  cuda_stream is a cudaStream_t (NULL = legacy default stream);
+ * allocator may be NULL.  Allocates the per-replica and per-instance state
+ * (about (N * (40 + 10 * K) + N * Bmax * 12 + 16 * log capacity + 160) bytes
+ * per replica).  On success *out receives the object and SIM_OK is returned;
+ * on failure *out is NULL and sim_last_error(NULL) describes the error. */
+int sim_create(const sim_cluster_t *cluster, const sim_tier_table_t *tiers, const sim_policy_t *policy,
+               void *cuda_stream, const sim_allocator_t *allocator, sim_t **out);
+
+/* Loads the request traces and resets every replica to t = 0.
+ * replica_offsets (host, [R + 1]): replica r owns trace records
+ * [replica_offsets[r], replica_offsets[r+1]); offsets[0] = 0, non-decreasing,
+ * at most 2^32 - 2 records per replica.  arrival_us, prompt_len, output_len,
+ * tier ([total] each, host or device per on_device): arrival times in
+ * microseconds from the replica's start, sorted non-decreasing within a
+ * replica (requests with equal times are dispatched tier-major, then in trace
+ * order), prompt length P >= 1 and output length O >= 1 in tokens with
+ * P + O <= min(M * T, 65536), and tier < the replica's K.  Violations return
+ * SIM_ERR_TRACE and leave no trace loaded.  Synchronises the stream. */
+int sim_load_trace(sim_t *sim, const int64_t *replica_offsets, const uint32_t *arrival_us,
+                   const uint16_t *prompt_len, const uint16_t *output_len, const uint8_t *tier, int on_device);
+
+/* Resets every replica of the loaded trace to t = 0 (asynchronous). */
+int sim_reset(sim_t *sim);
+
+/* Advances every unfinished replica by at most max_steps_per_replica steps
+ * (>= 1) in one persistent kernel launch; a later call resumes where this one
+ * stopped.  If num_unfinished (host) is non-NULL the call synchronises and
+ * stores the number of replicas not yet SIM_REPLICA_DONE; otherwise it
+ * returns as soon as the work is queued.  Returns SIM_ERR_STATE without a
+ * loaded trace. */
+int sim_run(sim_t *sim, int64_t max_steps_per_replica, int64_t *num_unfinished);
+
+/* Copies results out (host or device per on_device; any pointer may be NULL
+ * to skip that output) and synchronises the stream.
+ * per_request [total records], in trace order; per_replica [R];
+ * events [R * event_log_capacity]: replica r's first
+ * min(log_events, capacity) records start at r * capacity, in the order the
+ * simulation produced them. */
+int sim_metrics(sim_t *sim, sim_request_result_t *per_request, sim_replica_stats_t *per_replica,
+                sim_migration_event_t *events, int on_device);
+
+/* Releases everything the object owns (synchronises the stream first).
+ * NULL is ignored. */
+void sim_destroy(sim_t *sim);
+
+/* Text of the last error on this object, or of the last failed sim_create on
+ * this thread when sim is NULL.  Valid until the next call on the object. */
+const char *sim_last_error(const sim_t *sim);
+
+/* Static description of a return code. */
+const char *sim_strerror(int code);
+
+/* Device bytes the object holds (0 for NULL). */
+size_t sim_device_bytes(const sim_t *sim);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MTSIM_H */

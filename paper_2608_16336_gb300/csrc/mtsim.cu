@@ -1,0 +1,1408 @@
+// mtsim.cu -- batched simulation of the multi-tier Llumnix-style scheduler
+// ("Beyond Binary Priorities: Multi-Tier SLA Scheduling for LLM Serving",
+// Sec. 3) for sm_103a, behind the C ABI declared in mtsim.h.
+//
+// Execution model
+//   One warp simulates one replica.  A persistent grid pulls replicas from an
+//   atomic work counter.  While a warp owns a replica, the replica's instance
+//   state (per-instance scalars, per-(instance, tier) queue heads/tails and
+//   request counts, headroom table) lives in shared memory; it is written back
+//   to HBM when the warp stops (step limit or completion), so sim_run can be
+//   resumed.  Instances are spread over lanes in contiguous blocks of
+//   c = ceil(N/32) per lane, so "lowest lane" order is "lowest instance" order.
+//   Per-request state stays in HBM: the read-only trace (SoA), the 16-byte
+//   result record, the tokens generated so far and a doubly linked list node
+//   that threads waiting requests into their (instance, tier) FCFS bucket.
+//   Running requests occupy per-instance slot arrays (request id + one packed
+//   64-bit state word); a batch advance or batch formation touches an
+//   instance's slots with two slots per lane.
+//
+// Exactness
+//   Everything is integer.  Freeness F = (M - U) / max(B, 1) (Sec. 3.2 Eq. 1-2)
+//   is kept per instance as an order-preserving 32-bit key
+//   floor((M - U) * 4096 / max(B, 1)): for batch sizes up to 64, two distinct
+//   fractions differ by at least 1/4032, so the floored keys order every pair
+//   of freeness values exactly as the fractions do and equal fractions get
+//   equal keys.  The arg-max/arg-min of dispatch and migration pairing are
+//   therefore one warp __reduce_{max,min}_sync plus a ballot (lowest index on
+//   ties).  The migration threshold max F - min F >= theta is checked exactly
+//   by 64-bit cross-multiplication.
+//   Since free + sum(running blocks) + inbound reservation = M on every
+//   instance, M - U reduces to free - HoL demand - sum of present-tier
+//   headroom.
+//
+// Safety
+//   No kernel waits on another warp, block or launch: there are no spin
+//   loops.  Every loop is bounded by the trace length, the batch size, or the
+//   per-call step limit.  Index checks on queue links and slot positions turn
+//   an inconsistency into SIM_ERR_INTERNAL for that replica instead of an
+//   out-of-bounds access.
+#include "mtsim.h"
+
+#include <cuda_runtime.h>
+
+#include <climits>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+namespace mt {
+
+constexpr uint32_t kIdle = 0xFFFFFFFFu;
+constexpr uint32_t kNil = 0xFFFFFFFFu;
+constexpr uint32_t kFull = 0xFFFFFFFFu;
+constexpr uint64_t kInf64 = ~0ull;
+constexpr int kKeyScale = 4096;  // >= 64 * 63: exact order of fractions with denominators <= 64
+constexpr int kMaxKeyRange = 1 << 19;
+
+enum : int { MIG_NONE = 0, MIG_SRC = 1, MIG_DST = 2 };
+
+// Slot state word: ctx (P + g) | blocks << 16 | left (O - g) << 32 | tier << 48 | flags << 56.
+constexpr uint64_t kFirst = 1ull << 56;                     // first token not produced yet
+constexpr uint64_t kAdvance = 1ull - (1ull << 32);          // ctx + 1, left - 1
+__device__ __forceinline__ uint32_t s_ctx(uint64_t s) { return (uint32_t)s & 0xFFFFu; }
+__device__ __forceinline__ uint32_t s_blocks(uint64_t s) { return (uint32_t)(s >> 16) & 0xFFFFu; }
+__device__ __forceinline__ uint32_t s_left(uint64_t s) { return (uint32_t)(s >> 32) & 0xFFFFu; }
+__device__ __forceinline__ uint32_t s_tier(uint64_t s) { return (uint32_t)(s >> 48) & 0xFFu; }
+__device__ __forceinline__ uint64_t s_make(uint32_t ctx, uint32_t blocks, uint32_t left, uint32_t tier, bool first) {
+    return (uint64_t)ctx | ((uint64_t)blocks << 16) | ((uint64_t)left << 32) | ((uint64_t)tier << 48) |
+           (first ? kFirst : 0ull);
+}
+
+// Byte offsets of the per-replica state blob (identical in HBM and shared memory).
+struct Layout {
+    uint32_t busy, free_, resv, hol, hr, key, mreq, mcopied;  // [N] x 4 B
+    uint32_t wmask;                                           // [N] x 2 B
+    uint32_t nrun, nb, mrole, mpeer;                          // [N] x 1 B
+    uint32_t cnt;                                             // [N*K] x 2 B
+    uint32_t head, tail;                                      // [N*K] x 4 B
+    uint32_t h;                                               // [K] x 4 B
+    uint32_t bytes;
+};
+
+// Per-replica scalars persisted between sim_run calls.
+struct RepState {
+    uint32_t t, cursor, finished, log_events;
+    uint64_t next_tick, steps, iterations, member_iterations, events;
+    uint32_t migrations, preemptions, starts, aborts;
+    int32_t status;
+    uint32_t pad_[3];
+};
+
+struct Params {
+    int R, N, M, T, tshift, Bmax, K, c, S, C, enable_mig, theta_num, theta_den;
+    uint32_t interval;
+    long long base, a, b, max_steps;
+    Layout L;
+    const long long *offsets;
+    const uint32_t *arrival;
+    const uint16_t *plen, *olen;
+    const uint8_t *tier;
+    uint16_t *g;
+    uint2 *link;  // .x = next, .y = prev
+    sim_request_result_t *res;
+    unsigned char *blobs;
+    uint32_t *srid;
+    uint64_t *sst;
+    RepState *rep;
+    sim_migration_event_t *log;
+    int *work;
+};
+
+// Per-warp view of the replica being simulated.  Pointers into shared memory
+// for instance state, into HBM for request state; scalars are warp-uniform.
+struct Ctx {
+    uint32_t *busy, *mreq, *head, *tail;
+    int *free_, *resv, *hol, *hr, *key, *mcopied, *h;
+    uint16_t *wmask, *cnt;
+    uint8_t *nrun, *nb, *mrole, *mpeer;
+    const uint32_t *arrival;
+    const uint16_t *plen, *olen;
+    const uint8_t *tier;
+    uint16_t *g;
+    uint2 *link;
+    sim_request_result_t *res;
+    uint32_t *srid;
+    uint64_t *sst;
+    sim_migration_event_t *log;
+    int N, K, M, T, tshift, Bmax, S, C, c, lane;
+    uint32_t Q, t;
+};
+
+// Counters.  `finished` is warp-uniform; the others are exact on lane 0.
+struct Cnt {
+    uint32_t finished, log_events, migrations, preemptions, starts, aborts;
+    uint64_t steps, iterations, member_iterations, events;
+    int status;
+};
+
+__device__ __forceinline__ int blocks_for(const Ctx &x, uint32_t tokens) {
+    return x.tshift >= 0 ? (int)((tokens + (uint32_t)x.T - 1u) >> x.tshift)
+                         : (int)((tokens + (uint32_t)x.T - 1u) / (uint32_t)x.T);
+}
+
+__device__ __forceinline__ int make_key(int num, int nrun) {
+    const long long den = nrun > 0 ? nrun : 1;
+    const long long v = (long long)num * kKeyScale;
+    long long q = v / den;
+    if (v % den != 0 && v < 0) --q;
+    return (int)q;
+}
+
+__device__ __forceinline__ int fnum(const Ctx &x, int i) { return x.free_[i] - x.hol[i] - x.hr[i]; }
+
+__device__ __forceinline__ void set_key(const Ctx &x, int i) { x.key[i] = make_key(fnum(x, i), x.nrun[i]); }
+
+__device__ __forceinline__ void refresh_keys(const Ctx &x) {
+    for (int j = 0; j < x.c; ++j) {
+        const int i = x.lane * x.c + j;
+        if (i < x.N) set_key(x, i);
+    }
+    __syncwarp();
+}
+
+__device__ __forceinline__ uint32_t own_mask(const Ctx &x) {
+    uint32_t m = 0;
+    for (int j = 0; j < x.c; ++j)
+        if (x.lane * x.c + j < x.N) m |= 1u << j;
+    return m;
+}
+
+// Arg-max (want_max) or arg-min of the freeness key over the instances whose
+// bit is set in `el` (bit j = instance lane*c + j), excluding `excl`; lowest
+// index on ties; -1 if none.  Collective.
+__device__ __forceinline__ int arg_ext(const Ctx &x, uint32_t el, bool want_max, int excl) {
+    int bv = 0, bi = -1;
+    for (int j = 0; j < x.c; ++j) {
+        const int i = x.lane * x.c + j;
+        if (((el >> j) & 1u) && i != excl) {
+            const int k = x.key[i];
+            if (bi < 0 || (want_max ? k > bv : k < bv)) { bv = k; bi = i; }
+        }
+    }
+    const int v = bi >= 0 ? bv : (want_max ? INT_MIN : INT_MAX);
+    const int m = want_max ? __reduce_max_sync(kFull, v) : __reduce_min_sync(kFull, v);
+    const uint32_t eq = __ballot_sync(kFull, bi >= 0 && v == m);
+    if (!eq) return -1;
+    return __shfl_sync(kFull, bi, __ffs(eq) - 1);
+}
+
+// ---- lane-0 bookkeeping helpers (no collectives inside) --------------------
+__device__ __forceinline__ void cnt_inc(const Ctx &x, int i, int k) {
+    if (x.cnt[i * x.K + k]++ == 0) x.hr[i] += x.h[k];
+}
+__device__ __forceinline__ void cnt_dec(const Ctx &x, int i, int k) {
+    if (--x.cnt[i * x.K + k] == 0) x.hr[i] -= x.h[k];
+}
+__device__ __forceinline__ void push_back(const Ctx &x, int i, int k, uint32_t r) {
+    const int b = i * x.K + k;
+    const uint32_t tl = x.tail[b];
+    x.link[r] = make_uint2(kNil, tl);
+    if (tl != kNil) x.link[tl].x = r; else x.head[b] = r;
+    x.tail[b] = r;
+    x.wmask[i] |= (uint16_t)(1u << k);
+}
+__device__ __forceinline__ void push_front(const Ctx &x, int i, int k, uint32_t r) {
+    const int b = i * x.K + k;
+    const uint32_t hd = x.head[b];
+    x.link[r] = make_uint2(hd, kNil);
+    if (hd != kNil) x.link[hd].y = r; else x.tail[b] = r;
+    x.head[b] = r;
+    x.wmask[i] |= (uint16_t)(1u << k);
+}
+__device__ __forceinline__ uint32_t pop_front(const Ctx &x, int i, int k, Cnt &cn) {
+    const int b = i * x.K + k;
+    const uint32_t r = x.head[b];
+    if (r >= x.Q) { cn.status = SIM_ERR_INTERNAL; return kNil; }
+    const uint32_t nx = x.link[r].x;
+    x.head[b] = nx;
+    if (nx != kNil) x.link[nx].y = kNil;
+    else { x.tail[b] = kNil; x.wmask[i] &= (uint16_t)~(1u << k); }
+    return r;
+}
+__device__ __forceinline__ uint32_t pop_back(const Ctx &x, int i, int k, Cnt &cn) {
+    const int b = i * x.K + k;
+    const uint32_t r = x.tail[b];
+    if (r >= x.Q) { cn.status = SIM_ERR_INTERNAL; return kNil; }
+    const uint32_t pv = x.link[r].y;
+    x.tail[b] = pv;
+    if (pv != kNil) x.link[pv].x = kNil;
+    else { x.head[b] = kNil; x.wmask[i] &= (uint16_t)~(1u << k); }
+    return r;
+}
+// HoL demand: KV blocks the head of the highest-priority non-empty bucket needs.
+__device__ __forceinline__ void refresh_hol(const Ctx &x, int i) {
+    const uint32_t wm = x.wmask[i];
+    if (!wm) { x.hol[i] = 0; return; }
+    const uint32_t r = x.head[i * x.K + (__ffs(wm) - 1)];
+    x.hol[i] = blocks_for(x, (uint32_t)x.plen[r] + x.g[r]);
+}
+__device__ __forceinline__ void log_ev(const Ctx &x, Cnt &cn, int kind, uint32_t r, int s, int d, int blocks) {
+    const uint32_t k = cn.log_events++;
+    if (k < (uint32_t)x.C) {
+        uint4 w;
+        w.x = x.t;
+        w.y = r;
+        w.z = (uint32_t)(blocks & 0xFFFF) | ((uint32_t)s << 16) | ((uint32_t)d << 24);
+        w.w = (uint32_t)kind;
+        reinterpret_cast<uint4 *>(x.log)[k] = w;
+    }
+}
+__device__ __forceinline__ void bump_mig(const Ctx &x, uint32_t r) {
+    atomicAdd(reinterpret_cast<unsigned int *>(reinterpret_cast<unsigned char *>(x.res + r) + 12), 1u);
+}
+__device__ __forceinline__ void bump_pre(const Ctx &x, uint32_t r) {
+    atomicAdd(reinterpret_cast<unsigned int *>(reinterpret_cast<unsigned char *>(x.res + r) + 12), 1u << 16);
+}
+__device__ __forceinline__ void clear_mig(const Ctx &x, int s, int d) {
+    x.mrole[s] = MIG_NONE;
+    x.mrole[d] = MIG_NONE;
+    x.mreq[s] = kNil;
+    x.mcopied[s] = 0;
+}
+// Abandon the staged copy out of source s: the destination releases what was copied.
+__device__ void abort_mig(const Ctx &x, Cnt &cn, int s) {
+    const int d = x.mpeer[s];
+    const int cp = x.mcopied[s];
+    x.free_[d] += cp;
+    x.resv[d] -= cp;
+    log_ev(x, cn, SIM_EV_ABORT, x.mreq[s], s, d, cp);
+    cn.aborts++;
+    clear_mig(x, s, d);
+}
+
+// ---- collective steps -------------------------------------------------------
+struct Slots {
+    uint64_t a0, a1;
+    uint32_t r0, r1;
+    bool v0, v1;
+};
+
+__device__ __forceinline__ Slots load_slots(const Ctx &x, int i, int n) {
+    Slots s;
+    const uint64_t *st = x.sst + (size_t)i * x.Bmax;
+    const uint32_t *rd = x.srid + (size_t)i * x.Bmax;
+    const int i0 = 2 * x.lane, i1 = i0 + 1;
+    s.v0 = i0 < n;
+    s.v1 = i1 < n;
+    s.a0 = s.v0 ? st[i0] : 0ull;
+    s.r0 = s.v0 ? rd[i0] : kNil;
+    s.a1 = s.v1 ? st[i1] : 0ull;
+    s.r1 = s.v1 ? rd[i1] : kNil;
+    return s;
+}
+
+// Writes the slots whose keep flag is set at their compacted (stable) positions; returns the count.
+__device__ __forceinline__ int compact_slots(const Ctx &x, int i, const Slots &s, bool k0, bool k1) {
+    uint64_t *st = x.sst + (size_t)i * x.Bmax;
+    uint32_t *rd = x.srid + (size_t)i * x.Bmax;
+    const uint32_t q0 = __ballot_sync(kFull, k0), q1 = __ballot_sync(kFull, k1);
+    const uint32_t below = (1u << x.lane) - 1u;
+    const int p0 = __popc(q0 & below) + __popc(q1 & below);
+    const int p1 = p0 + (k0 ? 1 : 0);
+    __syncwarp();
+    if (k0) { st[p0] = s.a0; rd[p0] = s.r0; }
+    if (k1) { st[p1] = s.a1; rd[p1] = s.r1; }
+    __syncwarp();
+    return __popc(q0) + __popc(q1);
+}
+
+// Commit a fully copied running request from s to d (Sec. 3.5, Fig. 4).
+__device__ void commit_mig(const Ctx &x, Cnt &cn, int s, int d, int pos, uint64_t a, uint32_t rid, const Slots &sl,
+                           int n) {
+    uint64_t *st = x.sst + (size_t)s * x.Bmax;
+    uint32_t *rd = x.srid + (size_t)s * x.Bmax;
+    const int i0 = 2 * x.lane, i1 = i0 + 1;
+    __syncwarp();
+    if (sl.v0 && i0 > pos) { st[i0 - 1] = sl.a0; rd[i0 - 1] = sl.r0; }
+    if (sl.v1 && i1 > pos) { st[i1 - 1] = sl.a1; rd[i1 - 1] = sl.r1; }
+    __syncwarp();
+    if (x.lane == 0) {
+        const int nd = x.nrun[d];
+        x.sst[(size_t)d * x.Bmax + nd] = a;
+        x.srid[(size_t)d * x.Bmax + nd] = rid;
+        x.nrun[d] = (uint8_t)(nd + 1);
+        x.nrun[s] = (uint8_t)(n - 1);
+        const int blocks = (int)s_blocks(a);
+        x.free_[s] += blocks;
+        x.resv[d] -= x.mcopied[s];
+        const int tr = (int)s_tier(a);
+        cnt_dec(x, s, tr);
+        cnt_inc(x, d, tr);
+        bump_mig(x, rid);
+        cn.migrations++;
+        cn.events++;
+        log_ev(x, cn, SIM_EV_COMMIT, rid, s, d, blocks);
+        clear_mig(x, s, d);
+    }
+    __syncwarp();
+}
+
+// One copy stage at the end of an iteration of migration source s.
+__device__ void migration_stage(const Ctx &x, Cnt &cn, int s) {
+    const int d = x.mpeer[s];
+    const uint32_t rid = x.mreq[s];
+    const int n = x.nrun[s];
+    const Slots sl = load_slots(x, s, n);
+    const uint32_t h0 = __ballot_sync(kFull, sl.v0 && sl.r0 == rid);
+    const uint32_t h1 = __ballot_sync(kFull, sl.v1 && sl.r1 == rid);
+    if (!(h0 | h1)) {
+        if (x.lane == 0) cn.status = SIM_ERR_INTERNAL;
+        __syncwarp();
+        return;
+    }
+    const int l = __ffs(h0 | h1) - 1;
+    const int j = ((h0 >> l) & 1u) ? 0 : 1;
+    const uint64_t a = __shfl_sync(kFull, j ? sl.a1 : sl.a0, l);
+    const int pos = 2 * l + j;
+    const int blocks = (int)s_blocks(a);
+    int commit = 0;
+    if (x.lane == 0) {
+        const int cp = x.mcopied[s];
+        const int cc = min(x.S, blocks - cp);
+        if (x.free_[d] < cc) {
+            abort_mig(x, cn, s);
+        } else {
+            x.free_[d] -= cc;
+            x.resv[d] += cc;
+            x.mcopied[s] = cp + cc;
+            commit = (cp + cc == blocks) && ((int)x.nrun[d] < x.Bmax);
+        }
+    }
+    commit = __shfl_sync(kFull, commit, 0);
+    __syncwarp();
+    if (commit) commit_mig(x, cn, s, d, pos, a, rid, sl, n);
+}
+
+// Phase 1: the iteration of instance i ends at t (Sec. 2.1 prefill/decode token accounting).
+__device__ void complete_instance(const Ctx &x, Cnt &cn, int i) {
+    const int n = x.nrun[i], nb = x.nb[i];
+    uint64_t *st = x.sst + (size_t)i * x.Bmax;
+    Slots sl = load_slots(x, i, n);
+    const int i0 = 2 * x.lane, i1 = i0 + 1;
+    const bool b0 = i0 < nb, b1 = i1 < nb;
+    int firsts = 0;
+    if (b0) {
+        sl.a0 += kAdvance;
+        if (sl.a0 & kFirst) { sl.a0 &= ~kFirst; x.res[sl.r0].first_token_us = x.t; ++firsts; }
+    }
+    if (b1) {
+        sl.a1 += kAdvance;
+        if (sl.a1 & kFirst) { sl.a1 &= ~kFirst; x.res[sl.r1].first_token_us = x.t; ++firsts; }
+    }
+    const bool f0 = b0 && s_left(sl.a0) == 0, f1 = b1 && s_left(sl.a1) == 0;
+    const uint32_t m0 = __ballot_sync(kFull, f0), m1 = __ballot_sync(kFull, f1);
+    firsts = __reduce_add_sync(kFull, firsts);
+    if (!(m0 | m1)) {
+        if (b0) st[i0] = sl.a0;
+        if (b1) st[i1] = sl.a1;
+    } else {
+        if (f0) { x.res[sl.r0].finish_us = x.t; x.res[sl.r0].final_instance = (uint16_t)i; }
+        if (f1) { x.res[sl.r1].finish_us = x.t; x.res[sl.r1].final_instance = (uint16_t)i; }
+        uint32_t lanes = m0 | m1;
+        while (lanes) {  // finished requests in batch order
+            const int l = __ffs(lanes) - 1;
+            lanes &= lanes - 1;
+            for (int j = 0; j < 2; ++j) {
+                if (!(((j ? m1 : m0) >> l) & 1u)) continue;
+                const uint64_t a = __shfl_sync(kFull, j ? sl.a1 : sl.a0, l);
+                const uint32_t r = __shfl_sync(kFull, j ? sl.r1 : sl.r0, l);
+                if (x.lane == 0) {
+                    x.free_[i] += (int)s_blocks(a);
+                    cnt_dec(x, i, (int)s_tier(a));
+                    if (x.mrole[i] == MIG_SRC && x.mreq[i] == r) abort_mig(x, cn, i);
+                }
+                __syncwarp();
+            }
+        }
+        const int kept = compact_slots(x, i, sl, sl.v0 && !f0, sl.v1 && !f1);
+        const uint32_t nfin = __popc(m0) + __popc(m1);
+        cn.finished += nfin;
+        if (x.lane == 0) { x.nrun[i] = (uint8_t)kept; cn.events += nfin; }
+    }
+    if (x.lane == 0) {
+        x.nb[i] = 0;
+        x.busy[i] = kIdle;
+        cn.events += (uint32_t)firsts;
+    }
+    __syncwarp();
+    if (x.mrole[i] == MIG_SRC) migration_stage(x, cn, i);
+}
+
+// Dispatch one arriving request r of tier k with prompt length P (Sec. 3.4).
+__device__ void dispatch_one(const Ctx &x, Cnt &cn, uint32_t r, int k, uint32_t P, uint32_t all) {
+    const int best = arg_ext(x, all, true, -1);
+    if (x.lane == 0) {
+        const uint32_t old = x.wmask[best];
+        push_back(x, best, k, r);
+        cnt_inc(x, best, k);
+        if ((old & ((2u << k) - 1u)) == 0) x.hol[best] = blocks_for(x, P);  // becomes head of line
+        x.res[r].dispatch_instance = (uint16_t)best;
+        cn.events++;
+        set_key(x, best);
+    }
+    __syncwarp();
+}
+
+// Phase 2: arrivals at t, tier 0 first, FCFS (trace order) within a tier.
+__device__ void dispatch_phase(const Ctx &x, Cnt &cn, uint32_t &cursor, uint64_t &next_arr) {
+    refresh_keys(x);
+    const uint32_t all = own_mask(x);
+    const uint32_t idx = cursor + (uint32_t)x.lane;
+    const bool in = idx < x.Q;
+    const uint32_t av = in ? x.arrival[idx] : kNil;
+    const uint32_t eq = __ballot_sync(kFull, in && av == x.t);
+    if (eq != kFull) {
+        const int m = __popc(eq);  // arrivals are sorted, so eq is a prefix of the lanes
+        const bool mine = x.lane < m;
+        const uint32_t tr = mine ? x.tier[idx] : 0u;
+        const uint32_t P = mine ? x.plen[idx] : 0u;
+        uint32_t tm = __reduce_or_sync(kFull, mine ? (1u << tr) : 0u);
+        while (tm) {
+            const int k = __ffs(tm) - 1;
+            tm &= tm - 1;
+            uint32_t bits = __ballot_sync(kFull, mine && tr == (uint32_t)k);
+            while (bits) {
+                const int l = __ffs(bits) - 1;
+                bits &= bits - 1;
+                dispatch_one(x, cn, cursor + (uint32_t)l, k, __shfl_sync(kFull, P, l), all);
+            }
+        }
+        const uint32_t nxt = __shfl_sync(kFull, av, m);  // lane m holds the next arrival (or none)
+        cursor += (uint32_t)m;
+        next_arr = cursor < x.Q ? (uint64_t)nxt : kInf64;
+        return;
+    }
+    // More than 32 arrivals share this time: count them, then go tier by tier.
+    uint32_t m = 32;
+    for (;;) {
+        const uint32_t j2 = cursor + m + (uint32_t)x.lane;
+        const bool in2 = j2 < x.Q;
+        const uint32_t e2 = __ballot_sync(kFull, in2 && x.arrival[j2] == x.t);
+        m += (uint32_t)__popc(e2);
+        if (e2 != kFull) break;
+    }
+    for (int k = 0; k < x.K; ++k) {
+        for (uint32_t base = 0; base < m; base += 32) {
+            const uint32_t j2 = cursor + base + (uint32_t)x.lane;
+            const bool mine = base + (uint32_t)x.lane < m;
+            const uint32_t tr = mine ? x.tier[j2] : 0u;
+            const uint32_t P = mine ? x.plen[j2] : 0u;
+            uint32_t bits = __ballot_sync(kFull, mine && tr == (uint32_t)k);
+            while (bits) {
+                const int l = __ffs(bits) - 1;
+                bits &= bits - 1;
+                dispatch_one(x, cn, cursor + base + (uint32_t)l, k, __shfl_sync(kFull, P, l), all);
+            }
+        }
+    }
+    cursor += m;
+    next_arr = cursor < x.Q ? (uint64_t)x.arrival[cursor] : kInf64;
+}
+
+// Phase 3: periodic rebalancing between low- and high-freeness instances (Sec. 3.5).
+__device__ void migration_tick(const Ctx &x, Cnt &cn, int theta_num, int theta_den) {
+    refresh_keys(x);
+    uint32_t el = 0;
+    for (int j = 0; j < x.c; ++j) {
+        const int i = x.lane * x.c + j;
+        if (i < x.N && x.mrole[i] == MIG_NONE) el |= 1u << j;
+    }
+    for (;;) {
+        const int nel = __reduce_add_sync(kFull, __popc(el));
+        if (nel < 2) break;
+        const int s = arg_ext(x, el, false, -1);
+        const int d = arg_ext(x, el, true, s);
+        const long long ns = fnum(x, s), ds = max((int)x.nrun[s], 1);
+        const long long nd = fnum(x, d), dd = max((int)x.nrun[d], 1);
+        if ((long long)theta_den * (nd * ds - ns * dd) < (long long)theta_num * dd * ds) break;
+        const bool has_wait = x.wmask[s] != 0;
+        const int n_s = x.nrun[s];
+        __syncwarp();
+        int moved = 0;
+        if (has_wait) {
+            if (x.lane == 0) {
+                const int k = 31 - __clz((unsigned)x.wmask[s]);
+                const uint32_t r = pop_back(x, s, k, cn);
+                if (r != kNil) {
+                    refresh_hol(x, s);
+                    cnt_dec(x, s, k);
+                    const uint32_t old = x.wmask[d];
+                    push_back(x, d, k, r);
+                    cnt_inc(x, d, k);
+                    if ((old & ((2u << k) - 1u)) == 0) x.hol[d] = blocks_for(x, (uint32_t)x.plen[r] + x.g[r]);
+                    bump_mig(x, r);
+                    cn.migrations++;
+                    cn.events++;
+                    log_ev(x, cn, SIM_EV_QUEUED, r, s, d, 0);
+                }
+            }
+            moved = 1;
+        } else if (n_s > 0) {
+            // running candidate: lowest priority, then fewest blocks, then newest
+            const Slots sl = load_slots(x, s, n_s);
+            const int k0 = sl.v0 ? (int)((s_tier(sl.a0) << 16) | (0xFFFFu - s_blocks(sl.a0))) : -1;
+            const int k1 = sl.v1 ? (int)((s_tier(sl.a1) << 16) | (0xFFFFu - s_blocks(sl.a1))) : -1;
+            const int km = __reduce_max_sync(kFull, max(k0, k1));
+            const uint32_t c0 = (sl.v0 && k0 == km) ? sl.r0 : 0u, c1 = (sl.v1 && k1 == km) ? sl.r1 : 0u;
+            const uint32_t rid = __reduce_max_sync(kFull, max(c0, c1));
+            const int blocks = (int)(0xFFFFu - ((uint32_t)km & 0xFFFFu));
+            if (x.free_[d] >= blocks) {
+                if (x.lane == 0) {
+                    x.mrole[s] = MIG_SRC;
+                    x.mpeer[s] = (uint8_t)d;
+                    x.mreq[s] = rid;
+                    x.mcopied[s] = 0;
+                    x.mrole[d] = MIG_DST;
+                    x.mpeer[d] = (uint8_t)s;
+                    cn.starts++;
+                    log_ev(x, cn, SIM_EV_START, rid, s, d, blocks);
+                }
+                moved = 1;
+            }
+        }
+        if (x.lane == s / x.c) el &= ~(1u << (s % x.c));
+        if (moved && x.lane == d / x.c) el &= ~(1u << (d % x.c));
+        __syncwarp();
+    }
+}
+
+// Preemption of running request r (state word a) on instance i: recompute style.
+__device__ void preempt_book(const Ctx &x, Cnt &cn, int i, uint32_t r, uint64_t a) {
+    const int tr = (int)s_tier(a);
+    x.g[r] = (uint16_t)(x.olen[r] - s_left(a));
+    const uint32_t old = x.wmask[i];
+    push_front(x, i, tr, r);
+    if ((old & ((1u << tr) - 1u)) == 0) x.hol[i] = blocks_for(x, s_ctx(a));  // now head of line
+    bump_pre(x, r);
+    cn.preemptions++;
+    cn.events++;
+    if (x.mrole[i] == MIG_SRC && x.mreq[i] == r) abort_mig(x, cn, i);
+}
+
+// Phase 4: batch formation at idle instance i (Sec. 2.2 continuous batching).
+__device__ void form_batch(const Ctx &x, Cnt &cn, int i, long long base, long long a_us, long long b_us) {
+    int n = x.nrun[i];
+    int fr = x.free_[i];
+    uint64_t *st = x.sst + (size_t)i * x.Bmax;
+    uint32_t *rd = x.srid + (size_t)i * x.Bmax;
+    Slots sl = load_slots(x, i, n);
+    const int i0 = 2 * x.lane, i1 = i0 + 1;
+    const int d0 = sl.v0 ? max(0, blocks_for(x, s_ctx(sl.a0)) - (int)s_blocks(sl.a0)) : 0;
+    const int d1 = sl.v1 ? max(0, blocks_for(x, s_ctx(sl.a1)) - (int)s_blocks(sl.a1)) : 0;
+    const int total = __reduce_add_sync(kFull, d0 + d1);
+    if (total <= fr) {
+        // (i) every running request gets the KV growth it needs
+        if (total > 0) {
+            fr -= total;
+            if (d0) st[i0] = sl.a0 + ((uint64_t)d0 << 16);
+            if (d1) st[i1] = sl.a1 + ((uint64_t)d1 << 16);
+        }
+    } else {
+        // (i) grow in running order; when out of blocks, preempt the lowest
+        // priority, newest running request (possibly the one growing).
+        bool al0 = sl.v0, al1 = sl.v1;
+        for (int idx = 0; idx < n; ++idx) {
+            const int l = idx >> 1, j = idx & 1;
+            for (;;) {
+                if (!__shfl_sync(kFull, (int)(j ? al1 : al0), l)) break;
+                const uint64_t a = __shfl_sync(kFull, j ? sl.a1 : sl.a0, l);
+                const int def = blocks_for(x, s_ctx(a)) - (int)s_blocks(a);
+                if (def <= 0) break;
+                if (fr > 0) {
+                    const int gv = min(fr, def);
+                    fr -= gv;
+                    if (x.lane == l) {
+                        if (j) sl.a1 += (uint64_t)gv << 16; else sl.a0 += (uint64_t)gv << 16;
+                    }
+                    continue;
+                }
+                const int t0 = al0 ? (int)s_tier(sl.a0) : -1, t1 = al1 ? (int)s_tier(sl.a1) : -1;
+                const int tmax = __reduce_max_sync(kFull, max(t0, t1));
+                const uint32_t c0 = (al0 && t0 == tmax) ? sl.r0 : 0u, c1 = (al1 && t1 == tmax) ? sl.r1 : 0u;
+                const uint32_t rmax = __reduce_max_sync(kFull, max(c0, c1));
+                const uint32_t vm0 = __ballot_sync(kFull, al0 && t0 == tmax && sl.r0 == rmax);
+                const uint32_t vm1 = __ballot_sync(kFull, al1 && t1 == tmax && sl.r1 == rmax);
+                const int vl = vm0 ? __ffs(vm0) - 1 : __ffs(vm1) - 1;
+                const int vj = vm0 ? 0 : 1;
+                const uint64_t va = __shfl_sync(kFull, vj ? sl.a1 : sl.a0, vl);
+                fr += (int)s_blocks(va);
+                if (x.lane == vl) { if (vj) al1 = false; else al0 = false; }
+                if (x.lane == 0) preempt_book(x, cn, i, rmax, va);
+                __syncwarp();
+                if (vl == l && vj == j) break;
+            }
+        }
+        n = compact_slots(x, i, sl, al0, al1);
+    }
+    // (ii) admission in (tier, FCFS) order while the head of line fits; (iii) start the iteration.
+    if (x.lane == 0) {
+        const int n_decode = n;
+        long long prefill = 0;
+        int nr = n;
+        while (nr < x.Bmax) {
+            const uint32_t wm = x.wmask[i];
+            if (!wm) break;
+            const int need = x.hol[i];
+            if (need > fr) break;
+            const int k = __ffs(wm) - 1;
+            const uint32_t r = pop_front(x, i, k, cn);
+            if (r == kNil) break;
+            const uint32_t P = x.plen[r], O = x.olen[r], gg = x.g[r];
+            st[nr] = s_make(P + gg, (uint32_t)need, O - gg, (uint32_t)k, gg == 0);
+            rd[nr] = r;
+            ++nr;
+            fr -= need;
+            prefill += (long long)(P + gg);
+            refresh_hol(x, i);
+        }
+        x.nrun[i] = (uint8_t)nr;
+        x.free_[i] = fr;
+        if (nr > 0) {
+            const long long end = (long long)x.t + base + a_us * prefill + b_us * (long long)n_decode;
+            if (end > 0xFFFFFFFELL) {
+                cn.status = SIM_ERR_OVERFLOW;
+            } else {
+                x.busy[i] = (uint32_t)end;
+                x.nb[i] = (uint8_t)nr;
+                cn.iterations++;
+                cn.member_iterations += (uint64_t)nr;
+            }
+        }
+    }
+    __syncwarp();
+}
+
+__device__ __forceinline__ void copy_blob(unsigned char *dst, const unsigned char *src, uint32_t bytes, int lane) {
+    for (uint32_t o = (uint32_t)lane * 16u; o < bytes; o += 512u)
+        *reinterpret_cast<uint4 *>(dst + o) = *reinterpret_cast<const uint4 *>(src + o);
+}
+
+__device__ Ctx make_ctx(const Params &p, unsigned char *blob, int r, int lane) {
+    Ctx x;
+    const Layout &L = p.L;
+    x.busy = reinterpret_cast<uint32_t *>(blob + L.busy);
+    x.free_ = reinterpret_cast<int *>(blob + L.free_);
+    x.resv = reinterpret_cast<int *>(blob + L.resv);
+    x.hol = reinterpret_cast<int *>(blob + L.hol);
+    x.hr = reinterpret_cast<int *>(blob + L.hr);
+    x.key = reinterpret_cast<int *>(blob + L.key);
+    x.mreq = reinterpret_cast<uint32_t *>(blob + L.mreq);
+    x.mcopied = reinterpret_cast<int *>(blob + L.mcopied);
+    x.wmask = reinterpret_cast<uint16_t *>(blob + L.wmask);
+    x.nrun = blob + L.nrun;
+    x.nb = blob + L.nb;
+    x.mrole = blob + L.mrole;
+    x.mpeer = blob + L.mpeer;
+    x.cnt = reinterpret_cast<uint16_t *>(blob + L.cnt);
+    x.head = reinterpret_cast<uint32_t *>(blob + L.head);
+    x.tail = reinterpret_cast<uint32_t *>(blob + L.tail);
+    x.h = reinterpret_cast<int *>(blob + L.h);
+    const long long o = p.offsets[r];
+    x.Q = (uint32_t)(p.offsets[r + 1] - o);
+    x.arrival = p.arrival + o;
+    x.plen = p.plen + o;
+    x.olen = p.olen + o;
+    x.tier = p.tier + o;
+    x.g = p.g + o;
+    x.link = p.link + o;
+    x.res = p.res + o;
+    x.srid = p.srid + (size_t)r * p.N * p.Bmax;
+    x.sst = p.sst + (size_t)r * p.N * p.Bmax;
+    x.log = p.log + (size_t)r * p.C;
+    x.N = p.N;
+    x.K = p.K;
+    x.M = p.M;
+    x.T = p.T;
+    x.tshift = p.tshift;
+    x.Bmax = p.Bmax;
+    x.S = p.S;
+    x.C = p.C;
+    x.c = p.c;
+    x.lane = lane;
+    x.t = 0;
+    return x;
+}
+
+// The persistent simulation kernel: each warp repeatedly takes a replica and
+// advances it by up to p.max_steps event times.
+__global__ void __launch_bounds__(64) k_run(Params p) {
+    extern __shared__ __align__(16) unsigned char smem[];
+    const int lane = threadIdx.x & 31;
+    unsigned char *blob = smem + (size_t)(threadIdx.x >> 5) * p.L.bytes;
+    for (;;) {
+        int r = 0;
+        if (lane == 0) r = atomicAdd(p.work, 1);
+        r = __shfl_sync(kFull, r, 0);
+        if (r >= p.R) break;
+        const RepState rs = p.rep[r];
+        if (rs.status != SIM_REPLICA_RUNNING) continue;
+        unsigned char *gblob = p.blobs + (size_t)r * p.L.bytes;
+        copy_blob(blob, gblob, p.L.bytes, lane);
+        __syncwarp();
+        Ctx x = make_ctx(p, blob, r, lane);
+        Cnt cn;
+        cn.finished = rs.finished;
+        cn.log_events = rs.log_events;
+        cn.migrations = rs.migrations;
+        cn.preemptions = rs.preemptions;
+        cn.starts = rs.starts;
+        cn.aborts = rs.aborts;
+        cn.steps = rs.steps;
+        cn.iterations = rs.iterations;
+        cn.member_iterations = rs.member_iterations;
+        cn.events = rs.events;
+        cn.status = SIM_REPLICA_RUNNING;
+        uint32_t cursor = rs.cursor;
+        uint64_t next_tick = rs.next_tick;
+        uint64_t next_arr = cursor < x.Q ? (uint64_t)x.arrival[cursor] : kInf64;
+        x.t = rs.t;
+        long long here = 0;
+        for (;;) {
+            if (cn.finished == x.Q) { cn.status = SIM_REPLICA_DONE; break; }
+            if (here >= p.max_steps) break;
+            // a0: next event time
+            uint32_t mb = kIdle;
+            for (int j = 0; j < x.c; ++j) {
+                const int i = lane * x.c + j;
+                if (i < x.N) mb = min(mb, x.busy[i]);
+            }
+            const uint32_t tb = __reduce_min_sync(kFull, mb);
+            uint64_t tc = next_arr;
+            if (tb != kIdle && (uint64_t)tb < tc) tc = tb;
+            if (tc == kInf64) { cn.status = SIM_ERR_DEADLOCK; break; }
+            bool tick = false;
+            if (p.enable_mig && next_tick <= tc) { tc = next_tick; tick = true; }
+            x.t = (uint32_t)tc;
+            ++here;
+            ++cn.steps;
+            // 1. iteration ends, ascending instance index
+            if (tb == x.t) {
+                uint32_t hits = 0;
+                for (int j = 0; j < x.c; ++j) {
+                    const int i = lane * x.c + j;
+                    if (i < x.N && x.busy[i] == x.t) hits |= 1u << j;
+                }
+                uint32_t lanes = __ballot_sync(kFull, hits != 0);
+                while (lanes) {
+                    const int l = __ffs(lanes) - 1;
+                    lanes &= lanes - 1;
+                    uint32_t h = __shfl_sync(kFull, hits, l);
+                    while (h) {
+                        const int j = __ffs(h) - 1;
+                        h &= h - 1;
+                        complete_instance(x, cn, l * x.c + j);
+                    }
+                }
+            }
+            // 2. dispatch of arrivals at t
+            if (next_arr == (uint64_t)x.t) dispatch_phase(x, cn, cursor, next_arr);
+            // 3. migration tick
+            if (tick) {
+                next_tick += p.interval;
+                migration_tick(x, cn, p.theta_num, p.theta_den);
+            }
+            // 4. batch formation at idle instances with work, ascending index
+            {
+                uint32_t want = 0;
+                for (int j = 0; j < x.c; ++j) {
+                    const int i = lane * x.c + j;
+                    if (i < x.N && x.busy[i] == kIdle && (x.nrun[i] > 0 || x.wmask[i] != 0)) want |= 1u << j;
+                }
+                uint32_t lanes = __ballot_sync(kFull, want != 0);
+                while (lanes) {
+                    const int l = __ffs(lanes) - 1;
+                    lanes &= lanes - 1;
+                    uint32_t h = __shfl_sync(kFull, want, l);
+                    while (h) {
+                        const int j = __ffs(h) - 1;
+                        h &= h - 1;
+                        form_batch(x, cn, l * x.c + j, p.base, p.a, p.b);
+                    }
+                }
+            }
+            cn.status = __shfl_sync(kFull, cn.status, 0);
+            if (cn.status < 0) break;
+        }
+        __syncwarp();
+        copy_blob(gblob, blob, p.L.bytes, lane);
+        if (lane == 0) {
+            RepState o;
+            o.t = x.t;
+            o.cursor = cursor;
+            o.finished = cn.finished;
+            o.log_events = cn.log_events;
+            o.next_tick = next_tick;
+            o.steps = cn.steps;
+            o.iterations = cn.iterations;
+            o.member_iterations = cn.member_iterations;
+            o.events = cn.events;
+            o.migrations = cn.migrations;
+            o.preemptions = cn.preemptions;
+            o.starts = cn.starts;
+            o.aborts = cn.aborts;
+            o.status = cn.status;
+            o.pad_[0] = o.pad_[1] = o.pad_[2] = 0;
+            p.rep[r] = o;
+        }
+        __syncwarp();
+    }
+}
+
+// ---- set-up and export kernels ----------------------------------------------
+__global__ void k_init_state(Params p, const int *rep_table, const int *tbl_k, const int *tbl_h) {
+    const int lane = threadIdx.x & 31;
+    const int warps = (gridDim.x * blockDim.x) >> 5;
+    for (int r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < p.R; r += warps) {
+        unsigned char *b = p.blobs + (size_t)r * p.L.bytes;
+        const Layout &L = p.L;
+        const int N = p.N, NK = p.N * p.K;
+        const int tb = rep_table[r];
+        const int K = tbl_k[tb];
+        for (int i = lane; i < N; i += 32) {
+            reinterpret_cast<uint32_t *>(b + L.busy)[i] = kIdle;
+            reinterpret_cast<int *>(b + L.free_)[i] = p.M;
+            reinterpret_cast<int *>(b + L.resv)[i] = 0;
+            reinterpret_cast<int *>(b + L.hol)[i] = 0;
+            reinterpret_cast<int *>(b + L.hr)[i] = 0;
+            reinterpret_cast<int *>(b + L.key)[i] = 0;
+            reinterpret_cast<uint32_t *>(b + L.mreq)[i] = kNil;
+            reinterpret_cast<int *>(b + L.mcopied)[i] = 0;
+            reinterpret_cast<uint16_t *>(b + L.wmask)[i] = 0;
+            b[L.nrun + i] = 0;
+            b[L.nb + i] = 0;
+            b[L.mrole + i] = MIG_NONE;
+            b[L.mpeer + i] = 0;
+        }
+        for (int i = lane; i < NK; i += 32) {
+            reinterpret_cast<uint16_t *>(b + L.cnt)[i] = 0;
+            reinterpret_cast<uint32_t *>(b + L.head)[i] = kNil;
+            reinterpret_cast<uint32_t *>(b + L.tail)[i] = kNil;
+        }
+        for (int k = lane; k < p.K; k += 32)
+            reinterpret_cast<int *>(b + L.h)[k] = k < K ? tbl_h[tb * p.K + k] : 0;
+        if (lane == 0) {
+            RepState s;
+            memset(&s, 0, sizeof s);
+            s.next_tick = p.interval;
+            s.status = (p.offsets[r + 1] == p.offsets[r]) ? SIM_REPLICA_DONE : SIM_REPLICA_RUNNING;
+            p.rep[r] = s;
+        }
+    }
+}
+
+__global__ void k_init_requests(sim_request_result_t *res, uint16_t *g, long long n) {
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
+        reinterpret_cast<uint4 *>(res)[i] = make_uint4(0xFFFFFFFFu, kNil, kNil, 0u);
+        g[i] = 0;
+    }
+}
+
+// Trace validation: bit 0 unsorted, 1 tier >= K, 2 zero length, 3 too long, 4 bad arrival.
+__global__ void k_validate(const long long *offsets, int R, const uint32_t *arrival, const uint16_t *plen,
+                           const uint16_t *olen, const uint8_t *tier, const int *rep_table, const int *tbl_k,
+                           long long lim, long long n, int *flags) {
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
+        int lo = 0, hi = R - 1;  // replica r with offsets[r] <= i < offsets[r+1]
+        while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (offsets[mid] <= i) lo = mid; else hi = mid - 1;
+        }
+        int f = 0;
+        if (i > offsets[lo] && arrival[i] < arrival[i - 1]) f |= 1;
+        if ((int)tier[i] >= tbl_k[rep_table[lo]]) f |= 2;
+        if (plen[i] == 0 || olen[i] == 0) f |= 4;
+        if ((long long)plen[i] + olen[i] > lim) f |= 8;
+        if (arrival[i] == kNil) f |= 16;
+        if (f) atomicOr(flags, f);
+    }
+}
+
+__global__ void k_export_stats(const RepState *rep, sim_replica_stats_t *out, int R, int *unfinished) {
+    for (int r = blockIdx.x * blockDim.x + threadIdx.x; r < R; r += gridDim.x * blockDim.x) {
+        const RepState s = rep[r];
+        if (out) {
+            sim_replica_stats_t o;
+            o.steps = s.steps;
+            o.iterations = s.iterations;
+            o.member_iterations = s.member_iterations;
+            o.events = s.events;
+            o.migrations = s.migrations;
+            o.preemptions = s.preemptions;
+            o.migration_starts = s.starts;
+            o.migration_aborts = s.aborts;
+            o.log_events = s.log_events;
+            o.finished = s.finished;
+            o.last_time_us = s.t;
+            o.status = s.status;
+            out[r] = o;
+        }
+        if (unfinished && s.status != SIM_REPLICA_DONE) atomicAdd(unfinished, 1);
+    }
+}
+
+}  // namespace mt
+
+// ============================================================================
+// Host side: the C ABI.
+// ============================================================================
+struct sim {
+    sim_cluster_t cl;
+    sim_policy_t pol;
+    int K = 0, ntables = 0, c = 1, tshift = -1;
+    std::vector<int> tbl_k, tbl_h, rep_table;
+    cudaStream_t stream = nullptr;
+    sim_allocator_t al{};
+    bool use_al = false;
+    mt::Layout L{};
+    struct Buf { void *p; size_t n; };
+    std::vector<Buf> bufs;
+    size_t dev_bytes = 0;
+    int *d_rep_table = nullptr, *d_tbl_k = nullptr, *d_tbl_h = nullptr;
+    unsigned char *d_blobs = nullptr;
+    uint32_t *d_srid = nullptr;
+    uint64_t *d_sst = nullptr;
+    mt::RepState *d_rep = nullptr;
+    sim_migration_event_t *d_log = nullptr;
+    int *d_work = nullptr;  // [0] work counter, [1] validation flags, [2] unfinished count
+    int64_t qtot = 0, qcap = -1;
+    bool loaded = false;
+    std::vector<int64_t> h_off;
+    long long *d_off = nullptr;
+    uint32_t *d_arrival = nullptr;
+    uint16_t *d_plen = nullptr, *d_olen = nullptr, *d_g = nullptr;
+    uint8_t *d_tier = nullptr;
+    uint2 *d_link = nullptr;
+    sim_request_result_t *d_res = nullptr;
+    int sms = 0, grid = 0, wpb = 2;
+    size_t smem = 0;
+    std::string err;
+};
+
+namespace {
+
+thread_local std::string g_create_err;
+
+int fail(sim_t *s, int code, const char *fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    if (s) s->err = buf; else g_create_err = buf;
+    return code;
+}
+
+int cuda_fail(sim_t *s, cudaError_t e, const char *what) {
+    return fail(s, SIM_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+void *dalloc(sim_t *s, size_t n) {
+    if (n == 0) n = 16;
+    n = (n + 255) & ~(size_t)255;
+    void *p = nullptr;
+    if (s->use_al) {
+        p = s->al.alloc(s->al.ctx, n, (void *)s->stream);
+    } else if (cudaMallocAsync(&p, n, s->stream) != cudaSuccess) {
+        cudaGetLastError();
+        p = nullptr;
+    }
+    if (p) {
+        s->bufs.push_back({p, n});
+        s->dev_bytes += n;
+    }
+    return p;
+}
+
+void dfree(sim_t *s, void *p) {
+    if (!p) return;
+    for (size_t i = 0; i < s->bufs.size(); ++i) {
+        if (s->bufs[i].p == p) {
+            if (s->use_al) s->al.free(s->al.ctx, p, s->bufs[i].n, (void *)s->stream);
+            else cudaFreeAsync(p, s->stream);
+            s->dev_bytes -= s->bufs[i].n;
+            s->bufs.erase(s->bufs.begin() + i);
+            return;
+        }
+    }
+}
+
+mt::Layout make_layout(int N, int K) {
+    mt::Layout L;
+    uint32_t o = 0;
+    auto take = [&](uint32_t bytes, uint32_t align) {
+        o = (o + align - 1) / align * align;
+        const uint32_t at = o;
+        o += bytes;
+        return at;
+    };
+    L.busy = take(4u * N, 16);
+    L.free_ = take(4u * N, 16);
+    L.resv = take(4u * N, 16);
+    L.hol = take(4u * N, 16);
+    L.hr = take(4u * N, 16);
+    L.key = take(4u * N, 16);
+    L.mreq = take(4u * N, 16);
+    L.mcopied = take(4u * N, 16);
+    L.head = take(4u * N * K, 16);
+    L.tail = take(4u * N * K, 16);
+    L.h = take(4u * K, 16);
+    L.wmask = take(2u * N, 16);
+    L.cnt = take(2u * N * K, 16);
+    L.nrun = take(N, 16);
+    L.nb = take(N, 16);
+    L.mrole = take(N, 16);
+    L.mpeer = take(N, 16);
+    L.bytes = (o + 15u) & ~15u;
+    return L;
+}
+
+mt::Params make_params(const sim_t *s, long long max_steps) {
+    mt::Params p;
+    p.R = s->cl.num_replicas;
+    p.N = s->cl.num_instances;
+    p.M = s->cl.blocks_per_instance;
+    p.T = s->cl.tokens_per_block;
+    p.tshift = s->tshift;
+    p.Bmax = s->cl.max_batch;
+    p.K = s->K;
+    p.c = s->c;
+    p.S = s->pol.migrate_blocks_per_iter;
+    p.C = s->pol.event_log_capacity;
+    p.enable_mig = s->pol.enable_migration;
+    p.theta_num = s->pol.theta_num;
+    p.theta_den = s->pol.theta_den;
+    p.interval = (uint32_t)s->pol.migrate_interval_us;
+    p.base = s->pol.iter_base_us;
+    p.a = s->pol.iter_us_per_prefill_token;
+    p.b = s->pol.iter_us_per_decode_seq;
+    p.max_steps = max_steps;
+    p.L = s->L;
+    p.offsets = s->d_off;
+    p.arrival = s->d_arrival;
+    p.plen = s->d_plen;
+    p.olen = s->d_olen;
+    p.tier = s->d_tier;
+    p.g = s->d_g;
+    p.link = s->d_link;
+    p.res = s->d_res;
+    p.blobs = s->d_blobs;
+    p.srid = s->d_srid;
+    p.sst = s->d_sst;
+    p.rep = s->d_rep;
+    p.log = s->d_log;
+    p.work = s->d_work;
+    return p;
+}
+
+int check_launch(sim_t *s, const char *what) {
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_fail(s, e, what);
+    return SIM_OK;
+}
+
+int reset_state(sim_t *s) {
+    mt::Params p = make_params(s, 0);
+    const int R = s->cl.num_replicas;
+    const int blocks = (R + 7) / 8;
+    mt::k_init_state<<<blocks, 256, 0, s->stream>>>(p, s->d_rep_table, s->d_tbl_k, s->d_tbl_h);
+    int rc = check_launch(s, "k_init_state");
+    if (rc) return rc;
+    if (s->qtot > 0) {
+        const long long nb = std::min<long long>((s->qtot + 255) / 256, 65535LL * 16);
+        mt::k_init_requests<<<(unsigned)nb, 256, 0, s->stream>>>(s->d_res, s->d_g, (long long)s->qtot);
+        rc = check_launch(s, "k_init_requests");
+    }
+    return rc;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *sim_strerror(int code) {
+    switch (code) {
+        case SIM_OK: return "ok";
+        case SIM_ERR_ARG: return "invalid argument";
+        case SIM_ERR_TRACE: return "malformed trace";
+        case SIM_ERR_STATE: return "call out of order";
+        case SIM_ERR_OOM: return "device allocation failed";
+        case SIM_ERR_OVERFLOW: return "32-bit time or counter overflow";
+        case SIM_ERR_CUDA: return "CUDA runtime error";
+        case SIM_ERR_INTERNAL: return "device-side consistency check failed";
+        case SIM_ERR_DEADLOCK: return "no pending event while requests are unfinished";
+        default: return "unknown error";
+    }
+}
+
+const char *sim_last_error(const sim_t *s) { return s ? s->err.c_str() : g_create_err.c_str(); }
+
+size_t sim_device_bytes(const sim_t *s) { return s ? s->dev_bytes : 0; }
+
+int sim_create(const sim_cluster_t *cl, const sim_tier_table_t *tt, const sim_policy_t *pol, void *cuda_stream,
+               const sim_allocator_t *allocator, sim_t **out) {
+    if (!out) return fail(nullptr, SIM_ERR_ARG, "out is NULL");
+    *out = nullptr;
+    if (!cl || !tt || !pol) return fail(nullptr, SIM_ERR_ARG, "cluster, tiers and policy are required");
+    if (cl->num_replicas < 1) return fail(nullptr, SIM_ERR_ARG, "num_replicas must be >= 1");
+    if (cl->num_instances < 1 || cl->num_instances > SIM_MAX_INSTANCES)
+        return fail(nullptr, SIM_ERR_ARG, "num_instances must be in [1, %d]", SIM_MAX_INSTANCES);
+    if (cl->blocks_per_instance < 1 || cl->blocks_per_instance > SIM_MAX_BLOCKS)
+        return fail(nullptr, SIM_ERR_ARG, "blocks_per_instance must be in [1, %d]", SIM_MAX_BLOCKS);
+    if (cl->tokens_per_block < 1 || cl->tokens_per_block > 65535)
+        return fail(nullptr, SIM_ERR_ARG, "tokens_per_block must be in [1, 65535]");
+    if (cl->max_batch < 1 || cl->max_batch > SIM_MAX_BATCH)
+        return fail(nullptr, SIM_ERR_ARG, "max_batch must be in [1, %d]", SIM_MAX_BATCH);
+    if (tt->num_tables < 1 || tt->max_tiers < 1 || tt->max_tiers > SIM_MAX_TIERS)
+        return fail(nullptr, SIM_ERR_ARG, "need num_tables >= 1 and max_tiers in [1, %d]", SIM_MAX_TIERS);
+    if (!tt->num_tiers || !tt->headroom_blocks || !tt->replica_table)
+        return fail(nullptr, SIM_ERR_ARG, "tier table pointers must not be NULL");
+    for (int t = 0; t < tt->num_tables; ++t) {
+        const int K = tt->num_tiers[t];
+        if (K < 1 || K > tt->max_tiers) return fail(nullptr, SIM_ERR_ARG, "table %d: num_tiers out of range", t);
+        long long sum = 0;
+        for (int k = 0; k < K; ++k) {
+            const int h = tt->headroom_blocks[t * tt->max_tiers + k];
+            if (h < 0) return fail(nullptr, SIM_ERR_ARG, "table %d: negative headroom", t);
+            sum += h;
+        }
+        if (cl->blocks_per_instance + sum >= mt::kMaxKeyRange)
+            return fail(nullptr, SIM_ERR_ARG, "table %d: M + sum of headroom must be below 2^19", t);
+    }
+    for (int r = 0; r < cl->num_replicas; ++r)
+        if (tt->replica_table[r] < 0 || tt->replica_table[r] >= tt->num_tables)
+            return fail(nullptr, SIM_ERR_ARG, "replica %d: table index out of range", r);
+    if (pol->policy != SIM_POLICY_LLUMNIX_MT) return fail(nullptr, SIM_ERR_ARG, "unknown policy %d", pol->policy);
+    if (pol->enable_migration != 0 && pol->enable_migration != 1)
+        return fail(nullptr, SIM_ERR_ARG, "enable_migration must be 0 or 1");
+    const long long lim24 = 1LL << 24;
+    if (pol->iter_base_us < 0 || pol->iter_base_us > lim24 || pol->iter_us_per_prefill_token < 0 ||
+        pol->iter_us_per_prefill_token > lim24 || pol->iter_us_per_decode_seq < 0 || pol->iter_us_per_decode_seq > lim24)
+        return fail(nullptr, SIM_ERR_ARG, "iteration-time coefficients must be in [0, 2^24]");
+    if (pol->migrate_blocks_per_iter < 1 || pol->migrate_blocks_per_iter > 65535)
+        return fail(nullptr, SIM_ERR_ARG, "migrate_blocks_per_iter must be in [1, 65535]");
+    if (pol->theta_den < 1 || pol->theta_num < 0 || pol->theta_num > (1 << 20) || pol->theta_den > (1 << 20))
+        return fail(nullptr, SIM_ERR_ARG, "theta must be num/den with num in [0, 2^20], den in [1, 2^20]");
+    if (pol->event_log_capacity < 0 || pol->event_log_capacity > (1 << 24))
+        return fail(nullptr, SIM_ERR_ARG, "event_log_capacity must be in [0, 2^24]");
+    if (pol->migrate_interval_us < 1 || pol->migrate_interval_us > (1LL << 31))
+        return fail(nullptr, SIM_ERR_ARG, "migrate_interval_us must be in [1, 2^31]");
+    if (allocator && (!allocator->alloc || !allocator->free))
+        return fail(nullptr, SIM_ERR_ARG, "allocator needs both alloc and free");
+
+    sim_t *s = new (std::nothrow) sim_t();
+    if (!s) return fail(nullptr, SIM_ERR_OOM, "host allocation failed");
+    s->cl = *cl;
+    s->pol = *pol;
+    s->K = tt->max_tiers;
+    s->ntables = tt->num_tables;
+    s->tbl_k.assign(tt->num_tiers, tt->num_tiers + tt->num_tables);
+    s->tbl_h.assign(tt->headroom_blocks, tt->headroom_blocks + (size_t)tt->num_tables * tt->max_tiers);
+    s->rep_table.assign(tt->replica_table, tt->replica_table + cl->num_replicas);
+    s->stream = (cudaStream_t)cuda_stream;
+    if (allocator) { s->al = *allocator; s->use_al = true; }
+    s->c = (cl->num_instances + 31) / 32;
+    const int T = cl->tokens_per_block;
+    s->tshift = (T & (T - 1)) == 0 ? __builtin_ctz((unsigned)T) : -1;
+    s->L = make_layout(cl->num_instances, s->K);
+
+    const size_t R = (size_t)cl->num_replicas, N = (size_t)cl->num_instances, B = (size_t)cl->max_batch;
+    s->d_rep_table = (int *)dalloc(s, R * 4);
+    s->d_tbl_k = (int *)dalloc(s, (size_t)s->ntables * 4);
+    s->d_tbl_h = (int *)dalloc(s, (size_t)s->ntables * s->K * 4);
+    s->d_blobs = (unsigned char *)dalloc(s, R * s->L.bytes);
+    s->d_srid = (uint32_t *)dalloc(s, R * N * B * 4);
+    s->d_sst = (uint64_t *)dalloc(s, R * N * B * 8);
+    s->d_rep = (mt::RepState *)dalloc(s, R * sizeof(mt::RepState));
+    s->d_log = (sim_migration_event_t *)dalloc(s, R * (size_t)pol->event_log_capacity * sizeof(sim_migration_event_t));
+    s->d_work = (int *)dalloc(s, 16);
+    if (!s->d_rep_table || !s->d_tbl_k || !s->d_tbl_h || !s->d_blobs || !s->d_srid || !s->d_sst || !s->d_rep ||
+        !s->d_log || !s->d_work) {
+        const size_t held = s->dev_bytes;
+        sim_destroy(s);
+        return fail(nullptr, SIM_ERR_OOM, "device allocation failed (%zu bytes held when it failed)", held);
+    }
+    cudaError_t e = cudaMemcpyAsync(s->d_rep_table, s->rep_table.data(), R * 4, cudaMemcpyHostToDevice, s->stream);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(s->d_tbl_k, s->tbl_k.data(), (size_t)s->ntables * 4, cudaMemcpyHostToDevice, s->stream);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(s->d_tbl_h, s->tbl_h.data(), s->tbl_h.size() * 4, cudaMemcpyHostToDevice, s->stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s->stream);  // host vectors may be pageable
+    int dev = 0;
+    if (e == cudaSuccess) e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&s->sms, cudaDevAttrMultiProcessorCount, dev);
+    s->smem = (size_t)s->wpb * s->L.bytes;
+    if (e == cudaSuccess && s->smem > 48 * 1024)
+        e = cudaFuncSetAttribute(mt::k_run, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)s->smem);
+    int per_sm = 0;
+    if (e == cudaSuccess)
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, mt::k_run, 32 * s->wpb, s->smem);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        int rc = cuda_fail(nullptr, e, "sim_create");
+        sim_destroy(s);
+        return rc;
+    }
+    if (per_sm < 1) {
+        sim_destroy(s);
+        return fail(nullptr, SIM_ERR_ARG, "per-replica state (%u bytes) does not fit in shared memory", s->L.bytes);
+    }
+    const long long want = ((long long)R + s->wpb - 1) / s->wpb;
+    s->grid = (int)std::min<long long>(want, (long long)s->sms * per_sm);
+    *out = s;
+    return SIM_OK;
+}
+
+int sim_load_trace(sim_t *s, const int64_t *off, const uint32_t *arrival, const uint16_t *plen, const uint16_t *olen,
+                   const uint8_t *tier, int on_device) {
+    if (!s) return SIM_ERR_ARG;
+    if (!off) return fail(s, SIM_ERR_ARG, "replica_offsets is NULL");
+    const int R = s->cl.num_replicas;
+    if (off[0] != 0) return fail(s, SIM_ERR_TRACE, "replica_offsets[0] must be 0");
+    for (int r = 0; r < R; ++r) {
+        const int64_t q = off[r + 1] - off[r];
+        if (q < 0) return fail(s, SIM_ERR_TRACE, "replica_offsets must be non-decreasing (replica %d)", r);
+        if (q > (int64_t)0xFFFFFFFEll) return fail(s, SIM_ERR_TRACE, "replica %d has more than 2^32-2 records", r);
+    }
+    const int64_t n = off[R];
+    if (n > 0 && (!arrival || !plen || !olen || !tier)) return fail(s, SIM_ERR_ARG, "trace arrays must not be NULL");
+    s->loaded = false;
+    if (n > s->qcap) {
+        dfree(s, s->d_arrival); dfree(s, s->d_plen); dfree(s, s->d_olen); dfree(s, s->d_tier);
+        dfree(s, s->d_g); dfree(s, s->d_link); dfree(s, s->d_res);
+        s->d_arrival = nullptr; s->d_plen = s->d_olen = s->d_g = nullptr; s->d_tier = nullptr;
+        s->d_link = nullptr; s->d_res = nullptr;
+        s->qcap = -1;
+        const size_t m = (size_t)std::max<int64_t>(n, 1);
+        s->d_arrival = (uint32_t *)dalloc(s, m * 4);
+        s->d_plen = (uint16_t *)dalloc(s, m * 2);
+        s->d_olen = (uint16_t *)dalloc(s, m * 2);
+        s->d_tier = (uint8_t *)dalloc(s, m);
+        s->d_g = (uint16_t *)dalloc(s, m * 2);
+        s->d_link = (uint2 *)dalloc(s, m * 8);
+        s->d_res = (sim_request_result_t *)dalloc(s, m * 16);
+        if (!s->d_arrival || !s->d_plen || !s->d_olen || !s->d_tier || !s->d_g || !s->d_link || !s->d_res)
+            return fail(s, SIM_ERR_OOM, "device allocation for %lld trace records failed", (long long)n);
+        s->qcap = n;
+    }
+    if (!s->d_off) {
+        s->d_off = (long long *)dalloc(s, ((size_t)R + 1) * 8);
+        if (!s->d_off) return fail(s, SIM_ERR_OOM, "device allocation failed");
+    }
+    s->h_off.assign(off, off + R + 1);
+    const cudaMemcpyKind kind = on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
+    cudaError_t e = cudaMemcpyAsync(s->d_off, s->h_off.data(), ((size_t)R + 1) * 8, cudaMemcpyHostToDevice, s->stream);
+    if (n > 0) {
+        if (e == cudaSuccess) e = cudaMemcpyAsync(s->d_arrival, arrival, (size_t)n * 4, kind, s->stream);
+        if (e == cudaSuccess) e = cudaMemcpyAsync(s->d_plen, plen, (size_t)n * 2, kind, s->stream);
+        if (e == cudaSuccess) e = cudaMemcpyAsync(s->d_olen, olen, (size_t)n * 2, kind, s->stream);
+        if (e == cudaSuccess) e = cudaMemcpyAsync(s->d_tier, tier, (size_t)n, kind, s->stream);
+    }
+    if (e == cudaSuccess) e = cudaMemsetAsync(s->d_work, 0, 16, s->stream);
+    if (e != cudaSuccess) return cuda_fail(s, e, "sim_load_trace copy");
+    s->qtot = n;
+    if (n > 0) {
+        const long long lim = std::min<long long>((long long)s->cl.blocks_per_instance * s->cl.tokens_per_block, 65536);
+        const long long nb = std::min<long long>((n + 255) / 256, (long long)s->sms * 32);
+        mt::k_validate<<<(unsigned)std::max<long long>(nb, 1), 256, 0, s->stream>>>(
+            s->d_off, R, s->d_arrival, s->d_plen, s->d_olen, s->d_tier, s->d_rep_table, s->d_tbl_k, lim, n,
+            s->d_work + 1);
+        int rc = check_launch(s, "k_validate");
+        if (rc) return rc;
+    }
+    int flags = 0;
+    e = cudaMemcpyAsync(&flags, s->d_work + 1, 4, cudaMemcpyDeviceToHost, s->stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s->stream);
+    if (e != cudaSuccess) return cuda_fail(s, e, "sim_load_trace validation");
+    if (flags) {
+        return fail(s, SIM_ERR_TRACE, "malformed trace:%s%s%s%s%s", (flags & 1) ? " unsorted arrivals;" : "",
+                    (flags & 2) ? " tier >= K;" : "", (flags & 4) ? " zero prompt or output length;" : "",
+                    (flags & 8) ? " prompt + output longer than min(M*T, 65536);" : "",
+                    (flags & 16) ? " arrival time 0xFFFFFFFF;" : "");
+    }
+    int rc = reset_state(s);
+    if (rc) return rc;
+    s->loaded = true;
+    return SIM_OK;
+}
+
+int sim_reset(sim_t *s) {
+    if (!s) return SIM_ERR_ARG;
+    if (!s->loaded) return fail(s, SIM_ERR_STATE, "sim_reset before sim_load_trace");
+    return reset_state(s);
+}
+
+int sim_run(sim_t *s, int64_t max_steps, int64_t *num_unfinished) {
+    if (!s) return SIM_ERR_ARG;
+    if (!s->loaded) return fail(s, SIM_ERR_STATE, "sim_run before sim_load_trace");
+    if (max_steps < 1) return fail(s, SIM_ERR_ARG, "max_steps_per_replica must be >= 1");
+    cudaError_t e = cudaMemsetAsync(s->d_work, 0, 4, s->stream);
+    if (e != cudaSuccess) return cuda_fail(s, e, "sim_run");
+    mt::Params p = make_params(s, (long long)max_steps);
+    mt::k_run<<<s->grid, 32 * s->wpb, s->smem, s->stream>>>(p);
+    int rc = check_launch(s, "k_run");
+    if (rc) return rc;
+    if (num_unfinished) {
+        int cnt = 0;
+        e = cudaMemsetAsync(s->d_work + 2, 0, 4, s->stream);
+        if (e != cudaSuccess) return cuda_fail(s, e, "sim_run");
+        const int R = s->cl.num_replicas;
+        mt::k_export_stats<<<(R + 255) / 256, 256, 0, s->stream>>>(s->d_rep, nullptr, R, s->d_work + 2);
+        rc = check_launch(s, "k_export_stats");
+        if (rc) return rc;
+        e = cudaMemcpyAsync(&cnt, s->d_work + 2, 4, cudaMemcpyDeviceToHost, s->stream);
+        if (e == cudaSuccess) e = cudaStreamSynchronize(s->stream);
+        if (e != cudaSuccess) return cuda_fail(s, e, "sim_run");
+        *num_unfinished = cnt;
+    }
+    return SIM_OK;
+}
+
+int sim_metrics(sim_t *s, sim_request_result_t *per_request, sim_replica_stats_t *per_replica,
+                sim_migration_event_t *events, int on_device) {
+    if (!s) return SIM_ERR_ARG;
+    if (!s->loaded) return fail(s, SIM_ERR_STATE, "sim_metrics before sim_load_trace");
+    const cudaMemcpyKind kind = on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyDeviceToHost;
+    const int R = s->cl.num_replicas;
+    cudaError_t e = cudaSuccess;
+    if (per_request && s->qtot > 0)
+        e = cudaMemcpyAsync(per_request, s->d_res, (size_t)s->qtot * sizeof(sim_request_result_t), kind, s->stream);
+    if (e == cudaSuccess && per_replica) {
+        sim_replica_stats_t *dst = per_replica;
+        sim_replica_stats_t *tmp = nullptr;
+        if (!on_device) {
+            tmp = (sim_replica_stats_t *)dalloc(s, (size_t)R * sizeof(sim_replica_stats_t));
+            if (!tmp) return fail(s, SIM_ERR_OOM, "device allocation failed");
+            dst = tmp;
+        }
+        mt::k_export_stats<<<(R + 255) / 256, 256, 0, s->stream>>>(s->d_rep, dst, R, nullptr);
+        int rc = check_launch(s, "k_export_stats");
+        if (rc) return rc;
+        if (tmp) {
+            e = cudaMemcpyAsync(per_replica, tmp, (size_t)R * sizeof(sim_replica_stats_t), cudaMemcpyDeviceToHost,
+                                s->stream);
+            if (e == cudaSuccess) e = cudaStreamSynchronize(s->stream);
+            dfree(s, tmp);
+        }
+    }
+    if (e == cudaSuccess && events && s->pol.event_log_capacity > 0)
+        e = cudaMemcpyAsync(events, s->d_log, (size_t)R * s->pol.event_log_capacity * sizeof(sim_migration_event_t),
+                            kind, s->stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s->stream);
+    if (e != cudaSuccess) return cuda_fail(s, e, "sim_metrics");
+    return SIM_OK;
+}
+
+void sim_destroy(sim_t *s) {
+    if (!s) return;
+    cudaStreamSynchronize(s->stream);
+    while (!s->bufs.empty()) dfree(s, s->bufs.back().p);
+    cudaStreamSynchronize(s->stream);
+    cudaGetLastError();
+    delete s;
+}
+
+}  // extern "C"

@@ -278,10 +278,13 @@ CONFIG_NAMES = {
 }
 
 
-def config(cid: int, replicas=None, requests: int | None = None, nthreads: int | None = None) -> Workload:
+def config(cid: int, replicas=None, requests: int | None = None, nthreads: int | None = None,
+           seed_block: int = 0) -> Workload:
     """Builds workload ``cid`` (0..4).  ``replicas`` selects a subset of replica
     indices (their seeds are those of the full workload, so a subset is a true
-    sample of it); ``requests`` overrides the per-replica request count."""
+    sample of it); ``requests`` overrides the per-replica request count;
+    ``seed_block`` > 0 draws an independent copy of the workload (same shapes,
+    other seeds), e.g. one per GPU in a weak-scaling run."""
     T, BMAX = 16, 64
     if cid == 0:
         n, m, q = 4, 1024, 2000
@@ -337,7 +340,7 @@ def config(cid: int, replicas=None, requests: int | None = None, nthreads: int |
             tables_k.append(sp["k"])
             tables_h.append(h)
         rt.append(tables[key])
-        seed = 0 if cid == 0 else mix_seed(cid, i)
+        seed = (0 if cid == 0 else mix_seed(cid, i)) if seed_block == 0 else mix_seed(cid, (seed_block << 24) + i)
         params.append(_params(seed, qq, sp["k"], tier_probs(sp["dist"], sp["k"]), sp["rate"], sp["lens"], kind, cv))
         labels.append(sp["label"])
     off, arrival, plen, olen, tier = generate(params, nthreads)
