@@ -224,6 +224,43 @@ const char *sim_strerror(int code);
 /* Device bytes the object holds (0 for NULL). */
 size_t sim_device_bytes(const sim_t *sim);
 
+/* Scratch memory behind sim_run_static: one fixed device array per GPU. */
+#define SIM_STATIC_SCRATCH_BYTES (32u << 20)
+
+/* Allocation-free variant of a whole simulation (the paper has no
+ * counterpart; this is a library service).  For callers that cannot call
+ * cudaMalloc: code running inside a process whose device memory is entirely
+ * owned by another allocator or budget, plugins and hooks that must not touch
+ * the CUDA allocator at all, or contexts where an allocation's implicit
+ * synchronisation is not allowed.  It simulates every replica of the given
+ * trace from t = 0 to completion, exactly like sim_create + sim_load_trace +
+ * sim_run + sim_metrics, but allocates nothing: the simulation state lives in
+ * a file-scope device array of SIM_STATIC_SCRATCH_BYTES (32 MiB) that every
+ * GPU which loads the library holds until the process exits.
+ *
+ * cluster, tiers, policy: as for sim_create (host).  replica_offsets: host,
+ * [R + 1], as for sim_load_trace.  arrival_us, prompt_len, output_len, tier:
+ * DEVICE pointers to the trace, as for sim_load_trace.  per_request
+ * ([total records]) and per_replica ([R]) are DEVICE output buffers owned by
+ * the caller; events is a DEVICE buffer of R * policy->event_log_capacity
+ * records or NULL (then no log is written).  cuda_stream is a cudaStream_t
+ * (NULL = legacy default stream).
+ *
+ * Limits: the state of all replicas must fit in the scratch array, about
+ * R * (N * (40 + 10 * K) + N * Bmax * 12 + 100) + 10 * total records bytes;
+ * a larger problem returns SIM_ERR_ARG with the size it needed.  The first
+ * call on a device looks up the array's device address (cudaGetSymbolAddress)
+ * with that device current, so make the first call before any stream capture.
+ * Every call uses the same array and overwrites what the previous call left
+ * there; two calls whose work overlaps on the GPU (other streams, other host
+ * threads) race and corrupt each other's results.  Validates the trace
+ * (SIM_ERR_TRACE) and synchronises the stream before returning.  Errors are
+ * described by sim_last_error(NULL). */
+int sim_run_static(const sim_cluster_t *cluster, const sim_tier_table_t *tiers, const sim_policy_t *policy,
+                   const int64_t *replica_offsets, const uint32_t *arrival_us, const uint16_t *prompt_len,
+                   const uint16_t *output_len, const uint8_t *tier, sim_request_result_t *per_request,
+                   sim_replica_stats_t *per_replica, sim_migration_event_t *events, void *cuda_stream);
+
 #ifdef __cplusplus
 }
 #endif

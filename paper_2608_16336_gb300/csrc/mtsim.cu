@@ -1406,3 +1406,201 @@ void sim_destroy(sim_t *s) {
 }
 
 }  // extern "C"
+
+// ============================================================================
+// Allocation-free entry point: the whole simulation state in one file-scope
+// device array (see sim_run_static in mtsim.h).
+// ============================================================================
+static __device__ __align__(256) unsigned char g_static_scratch[SIM_STATIC_SCRATCH_BYTES];
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+void *g_static_scratch_addr[kMaxDevices];  // device address of g_static_scratch, looked up once per device
+
+int static_fail(int code, const char *fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    g_create_err = buf;
+    return code;
+}
+
+// The same limits sim_create enforces.
+int static_validate(const sim_cluster_t *cl, const sim_tier_table_t *tt, const sim_policy_t *pol) {
+    if (!cl || !tt || !pol) return static_fail(SIM_ERR_ARG, "cluster, tiers and policy are required");
+    if (cl->num_replicas < 1 || cl->num_instances < 1 || cl->num_instances > SIM_MAX_INSTANCES ||
+        cl->blocks_per_instance < 1 || cl->blocks_per_instance > SIM_MAX_BLOCKS || cl->tokens_per_block < 1 ||
+        cl->tokens_per_block > 65535 || cl->max_batch < 1 || cl->max_batch > SIM_MAX_BATCH)
+        return static_fail(SIM_ERR_ARG, "cluster shape out of range");
+    if (tt->num_tables < 1 || tt->max_tiers < 1 || tt->max_tiers > SIM_MAX_TIERS || !tt->num_tiers ||
+        !tt->headroom_blocks || !tt->replica_table)
+        return static_fail(SIM_ERR_ARG, "invalid tier tables");
+    for (int t = 0; t < tt->num_tables; ++t) {
+        const int K = tt->num_tiers[t];
+        if (K < 1 || K > tt->max_tiers) return static_fail(SIM_ERR_ARG, "table %d: num_tiers out of range", t);
+        long long sum = 0;
+        for (int k = 0; k < K; ++k) {
+            const int h = tt->headroom_blocks[t * tt->max_tiers + k];
+            if (h < 0) return static_fail(SIM_ERR_ARG, "table %d: negative headroom", t);
+            sum += h;
+        }
+        if (cl->blocks_per_instance + sum >= mt::kMaxKeyRange)
+            return static_fail(SIM_ERR_ARG, "table %d: M + sum of headroom must be below 2^19", t);
+    }
+    for (int r = 0; r < cl->num_replicas; ++r)
+        if (tt->replica_table[r] < 0 || tt->replica_table[r] >= tt->num_tables)
+            return static_fail(SIM_ERR_ARG, "replica %d: table index out of range", r);
+    const long long lim24 = 1LL << 24;
+    if (pol->policy != SIM_POLICY_LLUMNIX_MT || (pol->enable_migration != 0 && pol->enable_migration != 1) ||
+        pol->iter_base_us < 0 || pol->iter_base_us > lim24 || pol->iter_us_per_prefill_token < 0 ||
+        pol->iter_us_per_prefill_token > lim24 || pol->iter_us_per_decode_seq < 0 ||
+        pol->iter_us_per_decode_seq > lim24 || pol->migrate_blocks_per_iter < 1 ||
+        pol->migrate_blocks_per_iter > 65535 || pol->theta_den < 1 || pol->theta_num < 0 ||
+        pol->theta_num > (1 << 20) || pol->theta_den > (1 << 20) || pol->event_log_capacity < 0 ||
+        pol->event_log_capacity > (1 << 24) || pol->migrate_interval_us < 1 || pol->migrate_interval_us > (1LL << 31))
+        return static_fail(SIM_ERR_ARG, "policy out of range");
+    return SIM_OK;
+}
+
+size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+}  // namespace
+
+extern "C" int sim_run_static(const sim_cluster_t *cl, const sim_tier_table_t *tt, const sim_policy_t *pol,
+                              const int64_t *off, const uint32_t *arrival, const uint16_t *plen,
+                              const uint16_t *olen, const uint8_t *tier, sim_request_result_t *per_request,
+                              sim_replica_stats_t *per_replica, sim_migration_event_t *events, void *cuda_stream) {
+    int rc = static_validate(cl, tt, pol);
+    if (rc) return rc;
+    if (!off) return static_fail(SIM_ERR_ARG, "replica_offsets is NULL");
+    const int R = cl->num_replicas;
+    if (off[0] != 0) return static_fail(SIM_ERR_TRACE, "replica_offsets[0] must be 0");
+    for (int r = 0; r < R; ++r) {
+        const int64_t q = off[r + 1] - off[r];
+        if (q < 0 || q > (int64_t)0xFFFFFFFEll)
+            return static_fail(SIM_ERR_TRACE, "replica_offsets invalid at replica %d", r);
+    }
+    const int64_t n = off[R];
+    if (n > 0 && (!arrival || !plen || !olen || !tier || !per_request))
+        return static_fail(SIM_ERR_ARG, "trace and per_request pointers must not be NULL");
+    if (!per_replica) return static_fail(SIM_ERR_ARG, "per_replica must not be NULL");
+    const int cap = events ? pol->event_log_capacity : 0;
+
+    // Carve the scratch array.
+    const int N = cl->num_instances, B = cl->max_batch, K = tt->max_tiers;
+    const mt::Layout L = make_layout(N, K);
+    size_t o = 0;
+    const size_t o_blobs = o; o = align256(o + (size_t)R * L.bytes);
+    const size_t o_srid = o; o = align256(o + (size_t)R * N * B * 4);
+    const size_t o_sst = o; o = align256(o + (size_t)R * N * B * 8);
+    const size_t o_rep = o; o = align256(o + (size_t)R * sizeof(mt::RepState));
+    const size_t o_g = o; o = align256(o + (size_t)n * 2);
+    const size_t o_link = o; o = align256(o + (size_t)n * 8);
+    const size_t o_off = o; o = align256(o + ((size_t)R + 1) * 8);
+    const size_t o_rt = o; o = align256(o + (size_t)R * 4);
+    const size_t o_tk = o; o = align256(o + (size_t)tt->num_tables * 4);
+    const size_t o_th = o; o = align256(o + (size_t)tt->num_tables * K * 4);
+    const size_t o_work = o; o = align256(o + 16);
+    if (o > (size_t)SIM_STATIC_SCRATCH_BYTES)
+        return static_fail(SIM_ERR_ARG, "problem needs %zu bytes of scratch; sim_run_static holds %u bytes", o,
+                           (unsigned)SIM_STATIC_SCRATCH_BYTES);
+
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return static_fail(SIM_ERR_CUDA, "cudaGetDevice: %s", cudaGetErrorString(e));
+    if (dev < 0 || dev >= kMaxDevices) return static_fail(SIM_ERR_ARG, "device index %d not supported", dev);
+    if (!g_static_scratch_addr[dev]) {
+        void *p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_static_scratch);
+        if (e != cudaSuccess || !p)
+            return static_fail(SIM_ERR_CUDA, "cudaGetSymbolAddress: %s", cudaGetErrorString(e));
+        g_static_scratch_addr[dev] = p;
+    }
+    unsigned char *base = (unsigned char *)g_static_scratch_addr[dev];
+    cudaStream_t st = (cudaStream_t)cuda_stream;
+
+    mt::Params p;
+    memset(&p, 0, sizeof p);
+    p.R = R;
+    p.N = N;
+    p.M = cl->blocks_per_instance;
+    p.T = cl->tokens_per_block;
+    p.tshift = (p.T & (p.T - 1)) == 0 ? __builtin_ctz((unsigned)p.T) : -1;
+    p.Bmax = B;
+    p.K = K;
+    p.c = (N + 31) / 32;
+    p.S = pol->migrate_blocks_per_iter;
+    p.C = cap;
+    p.enable_mig = pol->enable_migration;
+    p.theta_num = pol->theta_num;
+    p.theta_den = pol->theta_den;
+    p.interval = (uint32_t)pol->migrate_interval_us;
+    p.base = pol->iter_base_us;
+    p.a = pol->iter_us_per_prefill_token;
+    p.b = pol->iter_us_per_decode_seq;
+    p.max_steps = 1LL << 62;
+    p.L = L;
+    p.offsets = (const long long *)(base + o_off);
+    p.arrival = arrival;
+    p.plen = plen;
+    p.olen = olen;
+    p.tier = tier;
+    p.g = (uint16_t *)(base + o_g);
+    p.link = (uint2 *)(base + o_link);
+    p.res = per_request;
+    p.blobs = base + o_blobs;
+    p.srid = (uint32_t *)(base + o_srid);
+    p.sst = (uint64_t *)(base + o_sst);
+    p.rep = (mt::RepState *)(base + o_rep);
+    p.log = events;
+    p.work = (int *)(base + o_work);
+    int *rt = (int *)(base + o_rt), *tk = (int *)(base + o_tk), *th = (int *)(base + o_th);
+
+    // Inputs the kernels read from device memory; the work counter and flags start at zero.
+    e = cudaMemcpyAsync((void *)p.offsets, off, ((size_t)R + 1) * 8, cudaMemcpyHostToDevice, st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(rt, tt->replica_table, (size_t)R * 4, cudaMemcpyHostToDevice, st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(tk, tt->num_tiers, (size_t)tt->num_tables * 4, cudaMemcpyHostToDevice, st);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(th, tt->headroom_blocks, (size_t)tt->num_tables * K * 4, cudaMemcpyHostToDevice, st);
+    if (e == cudaSuccess) e = cudaMemsetAsync(p.work, 0, 16, st);
+    if (e != cudaSuccess) return static_fail(SIM_ERR_CUDA, "sim_run_static copy: %s", cudaGetErrorString(e));
+    int sms = 0;
+    e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return static_fail(SIM_ERR_CUDA, "sim_run_static: %s", cudaGetErrorString(e));
+    if (n > 0) {
+        const long long lim = std::min<long long>((long long)p.M * p.T, 65536);
+        const long long nb = std::min<long long>((n + 255) / 256, (long long)sms * 32);
+        mt::k_validate<<<(unsigned)std::max<long long>(nb, 1), 256, 0, st>>>(p.offsets, R, arrival, plen, olen, tier,
+                                                                              rt, tk, lim, n, p.work + 1);
+        int flags = 0;
+        e = cudaGetLastError();
+        if (e == cudaSuccess) e = cudaMemcpyAsync(&flags, p.work + 1, 4, cudaMemcpyDeviceToHost, st);
+        if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+        if (e != cudaSuccess) return static_fail(SIM_ERR_CUDA, "sim_run_static validation: %s", cudaGetErrorString(e));
+        if (flags) return static_fail(SIM_ERR_TRACE, "malformed trace (validation flags 0x%x)", flags);
+    }
+    mt::k_init_state<<<(R + 7) / 8, 256, 0, st>>>(p, rt, tk, th);
+    if (n > 0) {
+        const long long nb = std::min<long long>((n + 255) / 256, 65535LL * 16);
+        mt::k_init_requests<<<(unsigned)nb, 256, 0, st>>>(per_request, p.g, (long long)n);
+    }
+    const int wpb = 2;
+    const size_t smem = (size_t)wpb * L.bytes;
+    e = cudaGetLastError();
+    if (e == cudaSuccess && smem > 48 * 1024)
+        e = cudaFuncSetAttribute(mt::k_run, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    int per_sm = 0;
+    if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, mt::k_run, 32 * wpb, smem);
+    if (e != cudaSuccess) return static_fail(SIM_ERR_CUDA, "sim_run_static launch set-up: %s", cudaGetErrorString(e));
+    if (per_sm < 1) return static_fail(SIM_ERR_ARG, "per-replica state does not fit in shared memory");
+    const int grid = (int)std::min<long long>(((long long)R + wpb - 1) / wpb, (long long)sms * per_sm);
+    mt::k_run<<<grid, 32 * wpb, smem, st>>>(p);
+    mt::k_export_stats<<<(R + 255) / 256, 256, 0, st>>>(p.rep, per_replica, R, nullptr);
+    e = cudaGetLastError();
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return static_fail(SIM_ERR_CUDA, "sim_run_static: %s", cudaGetErrorString(e));
+    return SIM_OK;
+}

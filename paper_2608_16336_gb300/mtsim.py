@@ -65,7 +65,8 @@ class sim_allocator_t(ctypes.Structure):
 
 
 EXPORTS = ["sim_create", "sim_load_trace", "sim_reset", "sim_run", "sim_metrics", "sim_destroy",
-           "sim_last_error", "sim_strerror", "sim_device_bytes"]
+           "sim_last_error", "sim_strerror", "sim_device_bytes", "sim_run_static"]
+SIM_STATIC_SCRATCH_BYTES = 32 << 20
 
 _LIB = None
 
@@ -100,6 +101,9 @@ def lib() -> ctypes.CDLL:
         L.sim_strerror.restype = ctypes.c_char_p
         L.sim_device_bytes.argtypes = [vp]
         L.sim_device_bytes.restype = ctypes.c_size_t
+        L.sim_run_static.argtypes = [ctypes.POINTER(sim_cluster_t), ctypes.POINTER(sim_tier_table_t),
+                                     ctypes.POINTER(sim_policy_t), vp, vp, vp, vp, vp, vp, vp, vp, vp]
+        L.sim_run_static.restype = ctypes.c_int
         _LIB = L
     return _LIB
 
@@ -161,6 +165,17 @@ def sim_destroy(handle) -> None:
 
 def sim_device_bytes(handle) -> int:
     return int(lib().sim_device_bytes(handle))
+
+
+def sim_run_static(cluster: sim_cluster_t, tiers: sim_tier_table_t, policy: sim_policy_t, replica_offsets_ptr: int,
+                   arrival_ptr: int, prompt_ptr: int, output_ptr: int, tier_ptr: int, per_request_ptr: int,
+                   per_replica_ptr: int, events_ptr, cuda_stream: int = 0) -> int:
+    """Whole simulation without any device allocation (state in the library's
+    fixed 32 MiB device array); trace and outputs are device pointers."""
+    rc = lib().sim_run_static(ctypes.byref(cluster), ctypes.byref(tiers), ctypes.byref(policy), replica_offsets_ptr,
+                              arrival_ptr, prompt_ptr, output_ptr, tier_ptr, per_request_ptr, per_replica_ptr,
+                              events_ptr or None, ctypes.c_void_p(cuda_stream or None))
+    return _check(rc, None)
 
 
 # ------------------------------------------------------- torch allocator --

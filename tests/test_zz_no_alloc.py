@@ -1,0 +1,96 @@
+"""The allocation-free entry point sim_run_static, for callers that cannot
+call cudaMalloc (their device memory belongs to another allocator or budget,
+or they run where an allocation is not allowed).  It must give exactly the
+results of the allocating path (sim_create ... sim_metrics), call after
+call, although every call reuses the same fixed device array."""
+import ctypes
+
+import numpy as np
+import pytest
+
+from paper_2608_16336_gb300 import mtsim
+from paper_2608_16336_gb300 import workloads as W
+from tests import parity
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def torch():
+    t = pytest.importorskip("torch")
+    if not t.cuda.is_available():
+        pytest.skip("no CUDA device")
+    t.cuda.set_device(0)
+    return t
+
+
+def _static_run(torch, w, cap):
+    """Runs w through sim_run_static with caller-owned device inputs and outputs."""
+    R = w.num_replicas
+    kmax = max(w.tables_k)
+    tk = np.asarray(w.tables_k, np.int32)
+    th = np.zeros((len(w.tables_k), kmax), np.int32)
+    for t, h in enumerate(w.tables_h):
+        th[t, : len(h)] = h
+    rt = np.ascontiguousarray(w.replica_table, np.int32)
+    cl = mtsim.sim_cluster_t(R, w.num_instances, w.blocks_per_instance, w.tokens_per_block, w.max_batch)
+    tt = mtsim.sim_tier_table_t(len(w.tables_k), kmax, tk.ctypes.data, th.ctypes.data, rt.ctypes.data)
+    pol = mtsim.sim_policy_t(0, w.enable_migration, w.iter_base_us, w.iter_us_per_prefill_token,
+                             w.iter_us_per_decode_seq, w.migrate_blocks_per_iter, w.theta_num, w.theta_den, cap,
+                             w.migrate_interval_us)
+    off = np.ascontiguousarray(w.offsets, np.int64)
+    dev = torch.device("cuda", 0)
+    tr = [torch.from_numpy(np.ascontiguousarray(a)).to(dev) for a in
+          (w.arrival_us.view(np.int32), w.prompt_len.view(np.int16), w.output_len.view(np.int16), w.tier)]
+    res = torch.empty(w.total_requests * 16, dtype=torch.uint8, device=dev)
+    st = torch.empty(R * 64, dtype=torch.uint8, device=dev)
+    ev = torch.empty(R * cap * 16, dtype=torch.uint8, device=dev)
+    torch.cuda.synchronize()
+    mtsim.sim_run_static(cl, tt, pol, off.ctypes.data, *[x.data_ptr() for x in tr], res.data_ptr(), st.data_ptr(),
+                         ev.data_ptr(), torch.cuda.current_stream().cuda_stream)
+    res_h = res.cpu().numpy().view(mtsim.RESULT_DTYPE)
+    st_h = st.cpu().numpy().view(mtsim.STATS_DTYPE)
+    ev_h = ev.cpu().numpy().view(mtsim.EVENT_DTYPE).reshape(R, cap)
+    events = []
+    for r in range(R):
+        n = min(int(st_h["log_events"][r]), cap)
+        e = ev_h[r, :n]
+        events.append(np.stack([e["time_us"], e["request"], e["src"], e["dst"], e["blocks"], e["kind"]],
+                               axis=1).astype(np.int64))
+    return res_h, st_h, events
+
+
+def test_static_entry_point_matches_allocating_path(torch):
+    cap = 2048
+    w = W.config(1, replicas=range(11), requests=2500)
+    want = parity.run_gpu(w, event_log_capacity=cap)
+    for _ in range(2):  # the second call reuses the scratch the first one left behind
+        got = _static_run(torch, w, cap)
+        assert (got[0] == want[0]).all()
+        assert (got[1] == want[1]).all()
+        for a, b in zip(got[2], want[2]):
+            assert (a == b).all()
+    # a different shape right after, on the same scratch
+    w0 = W.config(0, requests=500)
+    want0 = parity.run_gpu(w0, event_log_capacity=cap)
+    got0 = _static_run(torch, w0, cap)
+    assert (got0[0] == want0[0]).all() and (got0[1] == want0[1]).all()
+
+
+def test_static_entry_point_rejects_oversize(torch):
+    w = W.config(1, replicas=range(2), requests=10)
+    w.offsets = np.array([0, 10, 10 + 4_000_000], np.int64)  # 4M records need > 32 MiB of state
+    R = 2
+    tk = np.array([4], np.int32)
+    th = np.array([512, 256, 128, 64], np.int32)
+    rt = np.zeros(R, np.int32)
+    cl = mtsim.sim_cluster_t(R, 16, 2048, 16, 64)
+    tt = mtsim.sim_tier_table_t(1, 4, tk.ctypes.data, th.ctypes.data, rt.ctypes.data)
+    pol = mtsim.sim_policy_t(0, 1, 4000, 20, 30, 64, 3, 10, 0, 50000)
+    # real (small) device buffers: the size check must reject the call before any of them is used
+    small = [torch.zeros(64, dtype=torch.uint8, device="cuda") for _ in range(6)]
+    with pytest.raises(mtsim.SimError) as e:
+        mtsim.sim_run_static(cl, tt, pol, w.offsets.ctypes.data, *[x.data_ptr() for x in small], None,
+                             torch.cuda.current_stream().cuda_stream)
+    assert e.value.code == mtsim.SIM_ERR_ARG
+    assert "scratch" in str(e.value)
