@@ -6,16 +6,18 @@
 //   One warp simulates one replica.  A persistent grid pulls replicas from an
 //   atomic work counter.  While a warp owns a replica, the replica's instance
 //   state (per-instance scalars, per-(instance, tier) queue heads/tails and
-//   request counts, headroom table) lives in shared memory; it is written back
-//   to HBM when the warp stops (step limit or completion), so sim_run can be
-//   resumed.  Instances are spread over lanes in contiguous blocks of
-//   c = ceil(N/32) per lane, so "lowest lane" order is "lowest instance" order.
-//   Per-request state stays in HBM: the read-only trace (SoA), the 16-byte
-//   result record, the tokens generated so far and a doubly linked list node
-//   that threads waiting requests into their (instance, tier) FCFS bucket.
-//   Running requests occupy per-instance slot arrays (request id + one packed
-//   64-bit state word); a batch advance or batch formation touches an
-//   instance's slots with two slots per lane.
+//   request counts, headroom table) lives in shared memory, and so do the
+//   running-request slots when they fit; everything is written back to HBM
+//   when the warp stops (step limit or completion), so sim_run can be resumed.
+//   Instances are spread over lanes in contiguous blocks of C = ceil(N/32) per
+//   lane (C is a template parameter), so "lowest lane" order is "lowest
+//   instance" order.  Per-request state stays in HBM: the read-only trace
+//   (SoA), the 16-byte result record, the tokens generated so far and a doubly
+//   linked list node that threads waiting requests into their (instance, tier)
+//   FCFS bucket.  Running requests occupy per-instance slot arrays (request id
+//   + one packed 64-bit state word); a batch advance or batch formation touches
+//   an instance's slots as one 16-byte pair per lane.  The next 32 arrivals
+//   are held in registers, one per lane.
 //
 // Exactness
 //   Everything is integer.  Freeness F = (M - U) / max(B, 1) (Sec. 3.2 Eq. 1-2)
@@ -23,13 +25,15 @@
 //   floor((M - U) * 4096 / max(B, 1)): for batch sizes up to 64, two distinct
 //   fractions differ by at least 1/4032, so the floored keys order every pair
 //   of freeness values exactly as the fractions do and equal fractions get
-//   equal keys.  The arg-max/arg-min of dispatch and migration pairing are
-//   therefore one warp __reduce_{max,min}_sync plus a ballot (lowest index on
-//   ties).  The migration threshold max F - min F >= theta is checked exactly
-//   by 64-bit cross-multiplication.
-//   Since free + sum(running blocks) + inbound reservation = M on every
-//   instance, M - U reduces to free - HoL demand - sum of present-tier
-//   headroom.
+//   equal keys.  The floor division by B is the high half of the product
+//   with a per-block table entry ceil(2^64 / B), exact for every 32-bit
+//   numerator.  The
+//   arg-max/arg-min of dispatch and migration pairing are therefore one warp
+//   __reduce_{max,min}_sync plus a ballot (lowest index on ties).  The
+//   migration threshold max F - min F >= theta is checked exactly by 64-bit
+//   cross-multiplication.  Since free + sum(running blocks) + inbound
+//   reservation = M on every instance, M - U reduces to
+//   free - HoL demand - sum of present-tier headroom.
 //
 // Safety
 //   No kernel waits on another warp, block or launch: there are no spin
@@ -41,6 +45,7 @@
 
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <climits>
 #include <cstdarg>
 #include <cstdio>
@@ -51,25 +56,26 @@
 
 namespace mt {
 
-constexpr uint32_t kIdle = 0xFFFFFFFFu;
-constexpr uint32_t kNil = 0xFFFFFFFFu;
+constexpr uint32_t kNone = 0xFFFFFFFFu;  // idle instance / no pending event / nil link
 constexpr uint32_t kFull = 0xFFFFFFFFu;
-constexpr uint64_t kInf64 = ~0ull;
-constexpr int kKeyScale = 4096;  // >= 64 * 63: exact order of fractions with denominators <= 64
-constexpr int kMaxKeyRange = 1 << 19;
+constexpr int kKeyShift = 12;            // keys are floor(num * 4096 / den)
+constexpr int kMaxKeyRange = 1 << 19;    // |num| < 2^19 keeps num * 4096 below 2^31
+constexpr int kMagicShift = 40;          // floor(n / T) = (n * ceil(2^40 / T)) >> 40 for n < 2^20, T <= 65535
+constexpr int kWarpsPerBlock = 2;
+constexpr uint32_t kSmemSlotLimit = 24u * 1024u;  // slots go to shared memory up to this many bytes per replica
+constexpr uint32_t kMagicBytes = 528;             // ceil(2^64 / d) for d = 0..64, rounded up to 16 bytes
 
 enum : int { MIG_NONE = 0, MIG_SRC = 1, MIG_DST = 2 };
 
 // Slot state word: ctx (P + g) | blocks << 16 | left (O - g) << 32 | tier << 48 | flags << 56.
-constexpr uint64_t kFirst = 1ull << 56;                     // first token not produced yet
-constexpr uint64_t kAdvance = 1ull - (1ull << 32);          // ctx + 1, left - 1
+constexpr uint64_t kFirst = 1ull << 56;             // first token not produced yet
+constexpr uint64_t kAdvance = 1ull - (1ull << 32);  // ctx + 1, left - 1
 __device__ __forceinline__ uint32_t s_ctx(uint64_t s) { return (uint32_t)s & 0xFFFFu; }
-__device__ __forceinline__ uint32_t s_blocks(uint64_t s) { return (uint32_t)(s >> 16) & 0xFFFFu; }
+__device__ __forceinline__ uint32_t s_blocks(uint64_t s) { return (uint32_t)s >> 16; }
 __device__ __forceinline__ uint32_t s_left(uint64_t s) { return (uint32_t)(s >> 32) & 0xFFFFu; }
 __device__ __forceinline__ uint32_t s_tier(uint64_t s) { return (uint32_t)(s >> 48) & 0xFFu; }
 __device__ __forceinline__ uint64_t s_make(uint32_t ctx, uint32_t blocks, uint32_t left, uint32_t tier, bool first) {
-    return (uint64_t)ctx | ((uint64_t)blocks << 16) | ((uint64_t)left << 32) | ((uint64_t)tier << 48) |
-           (first ? kFirst : 0ull);
+    return (uint64_t)(ctx | (blocks << 16)) | ((uint64_t)(left | (tier << 16)) << 32) | (first ? kFirst : 0ull);
 }
 
 // Byte offsets of the per-replica state blob (identical in HBM and shared memory).
@@ -86,17 +92,21 @@ struct Layout {
 // Per-replica scalars persisted between sim_run calls.
 struct RepState {
     uint32_t t, cursor, finished, log_events;
-    uint64_t next_tick, steps, iterations, member_iterations, events;
+    uint32_t next_tick, pad0;
+    uint64_t steps, iterations, member_iterations, events;
     uint32_t migrations, preemptions, starts, aborts;
     int32_t status;
-    uint32_t pad_[3];
+    uint32_t pad1;
 };
 
 struct Params {
-    int R, N, M, T, tshift, Bmax, K, c, S, C, enable_mig, theta_num, theta_den;
-    uint32_t interval;
-    long long base, a, b, max_steps;
+    int R, N, M, T, Bmax, BP, K, S, cap, enable_mig, theta_num, theta_den;
+    uint32_t NS;                  // slots per replica: N * BP rounded up to a multiple of 4 (whole 16-byte rows)
+    uint32_t interval, max_steps;
+    unsigned long long magT;      // ceil(2^40 / T)
+    int base, a, b;
     Layout L;
+    uint32_t slot_bytes;          // NS * 12 when the slots live in shared memory, else 0
     const long long *offsets;
     const uint32_t *arrival;
     const uint16_t *plen, *olen;
@@ -113,79 +123,89 @@ struct Params {
 };
 
 // Per-warp view of the replica being simulated.  Pointers into shared memory
-// for instance state, into HBM for request state; scalars are warp-uniform.
+// for instance state (and slots when they fit), into HBM for request state;
+// scalars are warp-uniform.
 struct Ctx {
     uint32_t *busy, *mreq, *head, *tail;
     int *free_, *resv, *hol, *hr, *key, *mcopied, *h;
     uint16_t *wmask, *cnt;
     uint8_t *nrun, *nb, *mrole, *mpeer;
+    uint64_t *sst;
+    uint32_t *srid;
+    const unsigned long long *magic;  // [65]: ceil(2^64 / d) for d >= 2
     const uint32_t *arrival;
     const uint16_t *plen, *olen;
     const uint8_t *tier;
     uint16_t *g;
     uint2 *link;
     sim_request_result_t *res;
-    uint32_t *srid;
-    uint64_t *sst;
     sim_migration_event_t *log;
-    int N, K, M, T, tshift, Bmax, S, C, c, lane;
+    unsigned long long magT;
+    int N, K, T, Bmax, BP, S, cap, lane;
     uint32_t Q, t;
 };
 
 // Counters.  `finished` is warp-uniform; the others are exact on lane 0.
 struct Cnt {
-    uint32_t finished, log_events, migrations, preemptions, starts, aborts;
-    uint64_t steps, iterations, member_iterations, events;
+    uint32_t finished, log_events, migrations, preemptions, starts, aborts, steps, iterations;
+    uint64_t member_iterations, events;
     int status;
 };
 
 __device__ __forceinline__ int blocks_for(const Ctx &x, uint32_t tokens) {
-    return x.tshift >= 0 ? (int)((tokens + (uint32_t)x.T - 1u) >> x.tshift)
-                         : (int)((tokens + (uint32_t)x.T - 1u) / (uint32_t)x.T);
+    return (int)(((unsigned long long)(tokens + (uint32_t)x.T - 1u) * x.magT) >> kMagicShift);
 }
 
-__device__ __forceinline__ int make_key(int num, int nrun) {
-    const long long den = nrun > 0 ? nrun : 1;
-    const long long v = (long long)num * kKeyScale;
-    long long q = v / den;
-    if (v % den != 0 && v < 0) --q;
-    return (int)q;
+// floor(v / d) for v < 2^32 and 1 <= d <= 64: the high half of v * ceil(2^64 / d).
+__device__ __forceinline__ uint32_t div_small(const Ctx &x, uint32_t v, int d) {
+    return d == 1 ? v : (uint32_t)__umul64hi((unsigned long long)v, x.magic[d]);
+}
+
+__device__ __forceinline__ int make_key(const Ctx &x, int num, int nrun) {
+    const int d = nrun > 0 ? nrun : 1;
+    if (num >= 0) return (int)div_small(x, (uint32_t)num << kKeyShift, d);
+    return -(int)div_small(x, ((uint32_t)(-num) << kKeyShift) + (uint32_t)(d - 1), d);
 }
 
 __device__ __forceinline__ int fnum(const Ctx &x, int i) { return x.free_[i] - x.hol[i] - x.hr[i]; }
 
-__device__ __forceinline__ void set_key(const Ctx &x, int i) { x.key[i] = make_key(fnum(x, i), x.nrun[i]); }
+__device__ __forceinline__ void set_key(const Ctx &x, int i) { x.key[i] = make_key(x, fnum(x, i), x.nrun[i]); }
 
+template <int C>
 __device__ __forceinline__ void refresh_keys(const Ctx &x) {
-    for (int j = 0; j < x.c; ++j) {
-        const int i = x.lane * x.c + j;
+#pragma unroll
+    for (int j = 0; j < C; ++j) {
+        const int i = x.lane * C + j;
         if (i < x.N) set_key(x, i);
     }
     __syncwarp();
 }
 
+template <int C>
 __device__ __forceinline__ uint32_t own_mask(const Ctx &x) {
     uint32_t m = 0;
-    for (int j = 0; j < x.c; ++j)
-        if (x.lane * x.c + j < x.N) m |= 1u << j;
+#pragma unroll
+    for (int j = 0; j < C; ++j)
+        if (x.lane * C + j < x.N) m |= 1u << j;
     return m;
 }
 
 // Arg-max (want_max) or arg-min of the freeness key over the instances whose
-// bit is set in `el` (bit j = instance lane*c + j), excluding `excl`; lowest
+// bit is set in `el` (bit j = instance lane*C + j), excluding `excl`; lowest
 // index on ties; -1 if none.  Collective.
+template <int C>
 __device__ __forceinline__ int arg_ext(const Ctx &x, uint32_t el, bool want_max, int excl) {
-    int bv = 0, bi = -1;
-    for (int j = 0; j < x.c; ++j) {
-        const int i = x.lane * x.c + j;
+    int bv = want_max ? INT_MIN : INT_MAX, bi = -1;
+#pragma unroll
+    for (int j = 0; j < C; ++j) {
+        const int i = x.lane * C + j;
         if (((el >> j) & 1u) && i != excl) {
             const int k = x.key[i];
             if (bi < 0 || (want_max ? k > bv : k < bv)) { bv = k; bi = i; }
         }
     }
-    const int v = bi >= 0 ? bv : (want_max ? INT_MIN : INT_MAX);
-    const int m = want_max ? __reduce_max_sync(kFull, v) : __reduce_min_sync(kFull, v);
-    const uint32_t eq = __ballot_sync(kFull, bi >= 0 && v == m);
+    const int m = want_max ? __reduce_max_sync(kFull, bv) : __reduce_min_sync(kFull, bv);
+    const uint32_t eq = __ballot_sync(kFull, bi >= 0 && bv == m);
     if (!eq) return -1;
     return __shfl_sync(kFull, bi, __ffs(eq) - 1);
 }
@@ -200,37 +220,37 @@ __device__ __forceinline__ void cnt_dec(const Ctx &x, int i, int k) {
 __device__ __forceinline__ void push_back(const Ctx &x, int i, int k, uint32_t r) {
     const int b = i * x.K + k;
     const uint32_t tl = x.tail[b];
-    x.link[r] = make_uint2(kNil, tl);
-    if (tl != kNil) x.link[tl].x = r; else x.head[b] = r;
+    x.link[r] = make_uint2(kNone, tl);
+    if (tl != kNone) x.link[tl].x = r; else x.head[b] = r;
     x.tail[b] = r;
     x.wmask[i] |= (uint16_t)(1u << k);
 }
 __device__ __forceinline__ void push_front(const Ctx &x, int i, int k, uint32_t r) {
     const int b = i * x.K + k;
     const uint32_t hd = x.head[b];
-    x.link[r] = make_uint2(hd, kNil);
-    if (hd != kNil) x.link[hd].y = r; else x.tail[b] = r;
+    x.link[r] = make_uint2(hd, kNone);
+    if (hd != kNone) x.link[hd].y = r; else x.tail[b] = r;
     x.head[b] = r;
     x.wmask[i] |= (uint16_t)(1u << k);
 }
 __device__ __forceinline__ uint32_t pop_front(const Ctx &x, int i, int k, Cnt &cn) {
     const int b = i * x.K + k;
     const uint32_t r = x.head[b];
-    if (r >= x.Q) { cn.status = SIM_ERR_INTERNAL; return kNil; }
+    if (r >= x.Q) { cn.status = SIM_ERR_INTERNAL; return kNone; }
     const uint32_t nx = x.link[r].x;
     x.head[b] = nx;
-    if (nx != kNil) x.link[nx].y = kNil;
-    else { x.tail[b] = kNil; x.wmask[i] &= (uint16_t)~(1u << k); }
+    if (nx != kNone) x.link[nx].y = kNone;
+    else { x.tail[b] = kNone; x.wmask[i] &= (uint16_t)~(1u << k); }
     return r;
 }
 __device__ __forceinline__ uint32_t pop_back(const Ctx &x, int i, int k, Cnt &cn) {
     const int b = i * x.K + k;
     const uint32_t r = x.tail[b];
-    if (r >= x.Q) { cn.status = SIM_ERR_INTERNAL; return kNil; }
+    if (r >= x.Q) { cn.status = SIM_ERR_INTERNAL; return kNone; }
     const uint32_t pv = x.link[r].y;
     x.tail[b] = pv;
-    if (pv != kNil) x.link[pv].x = kNil;
-    else { x.head[b] = kNil; x.wmask[i] &= (uint16_t)~(1u << k); }
+    if (pv != kNone) x.link[pv].x = kNone;
+    else { x.head[b] = kNone; x.wmask[i] &= (uint16_t)~(1u << k); }
     return r;
 }
 // HoL demand: KV blocks the head of the highest-priority non-empty bucket needs.
@@ -242,7 +262,7 @@ __device__ __forceinline__ void refresh_hol(const Ctx &x, int i) {
 }
 __device__ __forceinline__ void log_ev(const Ctx &x, Cnt &cn, int kind, uint32_t r, int s, int d, int blocks) {
     const uint32_t k = cn.log_events++;
-    if (k < (uint32_t)x.C) {
+    if (k < (uint32_t)x.cap) {
         uint4 w;
         w.x = x.t;
         w.y = r;
@@ -260,11 +280,11 @@ __device__ __forceinline__ void bump_pre(const Ctx &x, uint32_t r) {
 __device__ __forceinline__ void clear_mig(const Ctx &x, int s, int d) {
     x.mrole[s] = MIG_NONE;
     x.mrole[d] = MIG_NONE;
-    x.mreq[s] = kNil;
+    x.mreq[s] = kNone;
     x.mcopied[s] = 0;
 }
 // Abandon the staged copy out of source s: the destination releases what was copied.
-__device__ void abort_mig(const Ctx &x, Cnt &cn, int s) {
+__device__ __forceinline__ void abort_mig(const Ctx &x, Cnt &cn, int s) {
     const int d = x.mpeer[s];
     const int cp = x.mcopied[s];
     x.free_[d] += cp;
@@ -275,6 +295,7 @@ __device__ void abort_mig(const Ctx &x, Cnt &cn, int s) {
 }
 
 // ---- collective steps -------------------------------------------------------
+// Lane l holds slots 2l and 2l+1 of an instance.
 struct Slots {
     uint64_t a0, a1;
     uint32_t r0, r1;
@@ -283,22 +304,30 @@ struct Slots {
 
 __device__ __forceinline__ Slots load_slots(const Ctx &x, int i, int n) {
     Slots s;
-    const uint64_t *st = x.sst + (size_t)i * x.Bmax;
-    const uint32_t *rd = x.srid + (size_t)i * x.Bmax;
-    const int i0 = 2 * x.lane, i1 = i0 + 1;
+    const int i0 = 2 * x.lane;
     s.v0 = i0 < n;
-    s.v1 = i1 < n;
-    s.a0 = s.v0 ? st[i0] : 0ull;
-    s.r0 = s.v0 ? rd[i0] : kNil;
-    s.a1 = s.v1 ? st[i1] : 0ull;
-    s.r1 = s.v1 ? rd[i1] : kNil;
+    s.v1 = i0 + 1 < n;
+    s.a0 = s.a1 = 0ull;
+    s.r0 = s.r1 = kNone;
+    if (s.v0) {
+        const ulonglong2 v = *reinterpret_cast<const ulonglong2 *>(x.sst + i * x.BP + i0);
+        const uint2 w = *reinterpret_cast<const uint2 *>(x.srid + i * x.BP + i0);
+        s.a0 = v.x;
+        s.a1 = v.y;
+        s.r0 = w.x;
+        s.r1 = w.y;
+    }
     return s;
+}
+
+__device__ __forceinline__ void store_states(const Ctx &x, int i, uint64_t a0, uint64_t a1) {
+    *reinterpret_cast<ulonglong2 *>(x.sst + i * x.BP + 2 * x.lane) = make_ulonglong2(a0, a1);
 }
 
 // Writes the slots whose keep flag is set at their compacted (stable) positions; returns the count.
 __device__ __forceinline__ int compact_slots(const Ctx &x, int i, const Slots &s, bool k0, bool k1) {
-    uint64_t *st = x.sst + (size_t)i * x.Bmax;
-    uint32_t *rd = x.srid + (size_t)i * x.Bmax;
+    uint64_t *st = x.sst + i * x.BP;
+    uint32_t *rd = x.srid + i * x.BP;
     const uint32_t q0 = __ballot_sync(kFull, k0), q1 = __ballot_sync(kFull, k1);
     const uint32_t below = (1u << x.lane) - 1u;
     const int p0 = __popc(q0 & below) + __popc(q1 & below);
@@ -311,10 +340,10 @@ __device__ __forceinline__ int compact_slots(const Ctx &x, int i, const Slots &s
 }
 
 // Commit a fully copied running request from s to d (Sec. 3.5, Fig. 4).
-__device__ void commit_mig(const Ctx &x, Cnt &cn, int s, int d, int pos, uint64_t a, uint32_t rid, const Slots &sl,
-                           int n) {
-    uint64_t *st = x.sst + (size_t)s * x.Bmax;
-    uint32_t *rd = x.srid + (size_t)s * x.Bmax;
+__device__ __forceinline__ void commit_mig(const Ctx &x, Cnt &cn, int s, int d, int pos, uint64_t a, uint32_t rid,
+                                           const Slots &sl, int n) {
+    uint64_t *st = x.sst + s * x.BP;
+    uint32_t *rd = x.srid + s * x.BP;
     const int i0 = 2 * x.lane, i1 = i0 + 1;
     __syncwarp();
     if (sl.v0 && i0 > pos) { st[i0 - 1] = sl.a0; rd[i0 - 1] = sl.r0; }
@@ -322,8 +351,8 @@ __device__ void commit_mig(const Ctx &x, Cnt &cn, int s, int d, int pos, uint64_
     __syncwarp();
     if (x.lane == 0) {
         const int nd = x.nrun[d];
-        x.sst[(size_t)d * x.Bmax + nd] = a;
-        x.srid[(size_t)d * x.Bmax + nd] = rid;
+        x.sst[d * x.BP + nd] = a;
+        x.srid[d * x.BP + nd] = rid;
         x.nrun[d] = (uint8_t)(nd + 1);
         x.nrun[s] = (uint8_t)(n - 1);
         const int blocks = (int)s_blocks(a);
@@ -342,7 +371,7 @@ __device__ void commit_mig(const Ctx &x, Cnt &cn, int s, int d, int pos, uint64_
 }
 
 // One copy stage at the end of an iteration of migration source s.
-__device__ void migration_stage(const Ctx &x, Cnt &cn, int s) {
+__device__ __forceinline__ void migration_stage(const Ctx &x, Cnt &cn, int s) {
     const int d = x.mpeer[s];
     const uint32_t rid = x.mreq[s];
     const int n = x.nrun[s];
@@ -378,34 +407,35 @@ __device__ void migration_stage(const Ctx &x, Cnt &cn, int s) {
 }
 
 // Phase 1: the iteration of instance i ends at t (Sec. 2.1 prefill/decode token accounting).
-__device__ void complete_instance(const Ctx &x, Cnt &cn, int i) {
+__device__ __forceinline__ void complete_instance(const Ctx &x, Cnt &cn, int i) {
     const int n = x.nrun[i], nb = x.nb[i];
-    uint64_t *st = x.sst + (size_t)i * x.Bmax;
     Slots sl = load_slots(x, i, n);
-    const int i0 = 2 * x.lane, i1 = i0 + 1;
-    const bool b0 = i0 < nb, b1 = i1 < nb;
-    int firsts = 0;
+    const int i0 = 2 * x.lane;
+    const bool b0 = i0 < nb, b1 = i0 + 1 < nb;
+    bool g0 = false, g1 = false;
     if (b0) {
         sl.a0 += kAdvance;
-        if (sl.a0 & kFirst) { sl.a0 &= ~kFirst; x.res[sl.r0].first_token_us = x.t; ++firsts; }
+        g0 = (sl.a0 & kFirst) != 0;
+        if (g0) { sl.a0 ^= kFirst; x.res[sl.r0].first_token_us = x.t; }
     }
     if (b1) {
         sl.a1 += kAdvance;
-        if (sl.a1 & kFirst) { sl.a1 &= ~kFirst; x.res[sl.r1].first_token_us = x.t; ++firsts; }
+        g1 = (sl.a1 & kFirst) != 0;
+        if (g1) { sl.a1 ^= kFirst; x.res[sl.r1].first_token_us = x.t; }
     }
     const bool f0 = b0 && s_left(sl.a0) == 0, f1 = b1 && s_left(sl.a1) == 0;
-    const uint32_t m0 = __ballot_sync(kFull, f0), m1 = __ballot_sync(kFull, f1);
-    firsts = __reduce_add_sync(kFull, firsts);
-    if (!(m0 | m1)) {
-        if (b0) st[i0] = sl.a0;
-        if (b1) st[i1] = sl.a1;
+    const uint32_t firsts = __reduce_add_sync(kFull, (uint32_t)g0 + (uint32_t)g1);
+    if (!__any_sync(kFull, f0 || f1)) {
+        if (b0) store_states(x, i, sl.a0, sl.a1);
     } else {
+        const uint32_t m0 = __ballot_sync(kFull, f0), m1 = __ballot_sync(kFull, f1);
         if (f0) { x.res[sl.r0].finish_us = x.t; x.res[sl.r0].final_instance = (uint16_t)i; }
         if (f1) { x.res[sl.r1].finish_us = x.t; x.res[sl.r1].final_instance = (uint16_t)i; }
         uint32_t lanes = m0 | m1;
         while (lanes) {  // finished requests in batch order
             const int l = __ffs(lanes) - 1;
             lanes &= lanes - 1;
+#pragma unroll
             for (int j = 0; j < 2; ++j) {
                 if (!(((j ? m1 : m0) >> l) & 1u)) continue;
                 const uint64_t a = __shfl_sync(kFull, j ? sl.a1 : sl.a0, l);
@@ -424,17 +454,17 @@ __device__ void complete_instance(const Ctx &x, Cnt &cn, int i) {
         if (x.lane == 0) { x.nrun[i] = (uint8_t)kept; cn.events += nfin; }
     }
     if (x.lane == 0) {
-        x.nb[i] = 0;
-        x.busy[i] = kIdle;
-        cn.events += (uint32_t)firsts;
+        x.busy[i] = kNone;
+        cn.events += firsts;
     }
     __syncwarp();
     if (x.mrole[i] == MIG_SRC) migration_stage(x, cn, i);
 }
 
 // Dispatch one arriving request r of tier k with prompt length P (Sec. 3.4).
-__device__ void dispatch_one(const Ctx &x, Cnt &cn, uint32_t r, int k, uint32_t P, uint32_t all) {
-    const int best = arg_ext(x, all, true, -1);
+template <int C>
+__device__ __forceinline__ void dispatch_one(const Ctx &x, Cnt &cn, uint32_t r, int k, uint32_t P, uint32_t all) {
+    const int best = arg_ext<C>(x, all, true, -1);
     if (x.lane == 0) {
         const uint32_t old = x.wmask[best];
         push_back(x, best, k, r);
@@ -447,75 +477,93 @@ __device__ void dispatch_one(const Ctx &x, Cnt &cn, uint32_t r, int k, uint32_t 
     __syncwarp();
 }
 
-// Phase 2: arrivals at t, tier 0 first, FCFS (trace order) within a tier.
-__device__ void dispatch_phase(const Ctx &x, Cnt &cn, uint32_t &cursor, uint64_t &next_arr) {
-    refresh_keys(x);
-    const uint32_t all = own_mask(x);
+// The next 32 trace records, one per lane: index pb + lane.
+struct ArrBuf {
+    uint32_t pb, time, tier, P;
+};
+
+__device__ __forceinline__ void arr_refill(const Ctx &x, ArrBuf &ab, uint32_t cursor) {
+    ab.pb = cursor;
     const uint32_t idx = cursor + (uint32_t)x.lane;
     const bool in = idx < x.Q;
-    const uint32_t av = in ? x.arrival[idx] : kNil;
-    const uint32_t eq = __ballot_sync(kFull, in && av == x.t);
+    ab.time = in ? x.arrival[idx] : kNone;
+    ab.tier = in ? (uint32_t)x.tier[idx] : 0u;
+    ab.P = in ? (uint32_t)x.plen[idx] : 0u;
+}
+
+// Phase 2: arrivals at t, tier 0 first, FCFS (trace order) within a tier.
+template <int C>
+__device__ __forceinline__ void dispatch_phase(const Ctx &x, Cnt &cn, uint32_t &cursor, uint32_t &next_arr,
+                                               ArrBuf &ab) {
+    refresh_keys<C>(x);
+    const uint32_t all = own_mask<C>(x);
+    const uint32_t off = cursor - ab.pb;
+    uint32_t eq = __ballot_sync(kFull, (uint32_t)x.lane >= off && ab.time == x.t);
+    if ((eq >> 31) && off > 0) {
+        // the run of arrivals at t may continue past the buffer: realign it on the cursor
+        arr_refill(x, ab, cursor);
+        eq = __ballot_sync(kFull, ab.time == x.t);
+    }
     if (eq != kFull) {
-        const int m = __popc(eq);  // arrivals are sorted, so eq is a prefix of the lanes
-        const bool mine = x.lane < m;
-        const uint32_t tr = mine ? x.tier[idx] : 0u;
-        const uint32_t P = mine ? x.plen[idx] : 0u;
-        uint32_t tm = __reduce_or_sync(kFull, mine ? (1u << tr) : 0u);
+        const bool mine = (eq >> x.lane) & 1u;
+        uint32_t tm = __reduce_or_sync(kFull, mine ? (1u << ab.tier) : 0u);
         while (tm) {
             const int k = __ffs(tm) - 1;
             tm &= tm - 1;
-            uint32_t bits = __ballot_sync(kFull, mine && tr == (uint32_t)k);
+            uint32_t bits = __ballot_sync(kFull, mine && ab.tier == (uint32_t)k);
             while (bits) {
                 const int l = __ffs(bits) - 1;
                 bits &= bits - 1;
-                dispatch_one(x, cn, cursor + (uint32_t)l, k, __shfl_sync(kFull, P, l), all);
+                dispatch_one<C>(x, cn, ab.pb + (uint32_t)l, k, __shfl_sync(kFull, ab.P, l), all);
             }
         }
-        const uint32_t nxt = __shfl_sync(kFull, av, m);  // lane m holds the next arrival (or none)
-        cursor += (uint32_t)m;
-        next_arr = cursor < x.Q ? (uint64_t)nxt : kInf64;
-        return;
-    }
-    // More than 32 arrivals share this time: count them, then go tier by tier.
-    uint32_t m = 32;
-    for (;;) {
-        const uint32_t j2 = cursor + m + (uint32_t)x.lane;
-        const bool in2 = j2 < x.Q;
-        const uint32_t e2 = __ballot_sync(kFull, in2 && x.arrival[j2] == x.t);
-        m += (uint32_t)__popc(e2);
-        if (e2 != kFull) break;
-    }
-    for (int k = 0; k < x.K; ++k) {
-        for (uint32_t base = 0; base < m; base += 32) {
-            const uint32_t j2 = cursor + base + (uint32_t)x.lane;
-            const bool mine = base + (uint32_t)x.lane < m;
-            const uint32_t tr = mine ? x.tier[j2] : 0u;
-            const uint32_t P = mine ? x.plen[j2] : 0u;
-            uint32_t bits = __ballot_sync(kFull, mine && tr == (uint32_t)k);
-            while (bits) {
-                const int l = __ffs(bits) - 1;
-                bits &= bits - 1;
-                dispatch_one(x, cn, cursor + base + (uint32_t)l, k, __shfl_sync(kFull, P, l), all);
+        cursor += (uint32_t)__popc(eq);
+    } else {
+        // 32 or more arrivals share this time (the buffer starts at the cursor):
+        // count them, then go tier by tier from the trace.
+        uint32_t m = 32;
+        for (;;) {
+            const uint32_t j2 = cursor + m + (uint32_t)x.lane;
+            const bool in2 = j2 < x.Q;
+            const uint32_t e2 = __ballot_sync(kFull, in2 && x.arrival[j2] == x.t);
+            m += (uint32_t)__popc(e2);
+            if (e2 != kFull) break;
+        }
+        for (int k = 0; k < x.K; ++k) {
+            for (uint32_t base = 0; base < m; base += 32) {
+                const uint32_t j2 = cursor + base + (uint32_t)x.lane;
+                const bool mine = base + (uint32_t)x.lane < m;
+                const uint32_t tr = mine ? x.tier[j2] : 0u;
+                const uint32_t P = mine ? x.plen[j2] : 0u;
+                uint32_t bits = __ballot_sync(kFull, mine && tr == (uint32_t)k);
+                while (bits) {
+                    const int l = __ffs(bits) - 1;
+                    bits &= bits - 1;
+                    dispatch_one<C>(x, cn, cursor + base + (uint32_t)l, k, __shfl_sync(kFull, P, l), all);
+                }
             }
         }
+        cursor += m;
     }
-    cursor += m;
-    next_arr = cursor < x.Q ? (uint64_t)x.arrival[cursor] : kInf64;
+    if (cursor - ab.pb >= 32u) arr_refill(x, ab, cursor);
+    next_arr = __shfl_sync(kFull, ab.time, (int)(cursor - ab.pb));
 }
 
 // Phase 3: periodic rebalancing between low- and high-freeness instances (Sec. 3.5).
-__device__ void migration_tick(const Ctx &x, Cnt &cn, int theta_num, int theta_den) {
-    refresh_keys(x);
+template <int C>
+__device__ __forceinline__ void migration_tick(const Ctx &x, Cnt &cn, int theta_num, int theta_den) {
+    refresh_keys<C>(x);
     uint32_t el = 0;
-    for (int j = 0; j < x.c; ++j) {
-        const int i = x.lane * x.c + j;
+#pragma unroll
+    for (int j = 0; j < C; ++j) {
+        const int i = x.lane * C + j;
         if (i < x.N && x.mrole[i] == MIG_NONE) el |= 1u << j;
     }
     for (;;) {
         const int nel = __reduce_add_sync(kFull, __popc(el));
         if (nel < 2) break;
-        const int s = arg_ext(x, el, false, -1);
-        const int d = arg_ext(x, el, true, s);
+        const int s = arg_ext<C>(x, el, false, -1);
+        const int d = arg_ext<C>(x, el, true, s);
         const long long ns = fnum(x, s), ds = max((int)x.nrun[s], 1);
         const long long nd = fnum(x, d), dd = max((int)x.nrun[d], 1);
         if ((long long)theta_den * (nd * ds - ns * dd) < (long long)theta_num * dd * ds) break;
@@ -527,7 +575,7 @@ __device__ void migration_tick(const Ctx &x, Cnt &cn, int theta_num, int theta_d
             if (x.lane == 0) {
                 const int k = 31 - __clz((unsigned)x.wmask[s]);
                 const uint32_t r = pop_back(x, s, k, cn);
-                if (r != kNil) {
+                if (r != kNone) {
                     refresh_hol(x, s);
                     cnt_dec(x, s, k);
                     const uint32_t old = x.wmask[d];
@@ -564,14 +612,14 @@ __device__ void migration_tick(const Ctx &x, Cnt &cn, int theta_num, int theta_d
                 moved = 1;
             }
         }
-        if (x.lane == s / x.c) el &= ~(1u << (s % x.c));
-        if (moved && x.lane == d / x.c) el &= ~(1u << (d % x.c));
+        if (x.lane == s / C) el &= ~(1u << (s % C));
+        if (moved && x.lane == d / C) el &= ~(1u << (d % C));
         __syncwarp();
     }
 }
 
 // Preemption of running request r (state word a) on instance i: recompute style.
-__device__ void preempt_book(const Ctx &x, Cnt &cn, int i, uint32_t r, uint64_t a) {
+__device__ __forceinline__ void preempt_book(const Ctx &x, Cnt &cn, int i, uint32_t r, uint64_t a) {
     const int tr = (int)s_tier(a);
     x.g[r] = (uint16_t)(x.olen[r] - s_left(a));
     const uint32_t old = x.wmask[i];
@@ -584,13 +632,10 @@ __device__ void preempt_book(const Ctx &x, Cnt &cn, int i, uint32_t r, uint64_t 
 }
 
 // Phase 4: batch formation at idle instance i (Sec. 2.2 continuous batching).
-__device__ void form_batch(const Ctx &x, Cnt &cn, int i, long long base, long long a_us, long long b_us) {
+__device__ __forceinline__ void form_batch(const Ctx &x, Cnt &cn, int i, int base, int a_us, int b_us) {
     int n = x.nrun[i];
     int fr = x.free_[i];
-    uint64_t *st = x.sst + (size_t)i * x.Bmax;
-    uint32_t *rd = x.srid + (size_t)i * x.Bmax;
     Slots sl = load_slots(x, i, n);
-    const int i0 = 2 * x.lane, i1 = i0 + 1;
     const int d0 = sl.v0 ? max(0, blocks_for(x, s_ctx(sl.a0)) - (int)s_blocks(sl.a0)) : 0;
     const int d1 = sl.v1 ? max(0, blocks_for(x, s_ctx(sl.a1)) - (int)s_blocks(sl.a1)) : 0;
     const int total = __reduce_add_sync(kFull, d0 + d1);
@@ -598,8 +643,7 @@ __device__ void form_batch(const Ctx &x, Cnt &cn, int i, long long base, long lo
         // (i) every running request gets the KV growth it needs
         if (total > 0) {
             fr -= total;
-            if (d0) st[i0] = sl.a0 + ((uint64_t)d0 << 16);
-            if (d1) st[i1] = sl.a1 + ((uint64_t)d1 << 16);
+            if (d0 | d1) store_states(x, i, sl.a0 + ((uint64_t)d0 << 16), sl.a1 + ((uint64_t)d1 << 16));
         }
     } else {
         // (i) grow in running order; when out of blocks, preempt the lowest
@@ -641,7 +685,7 @@ __device__ void form_batch(const Ctx &x, Cnt &cn, int i, long long base, long lo
     // (ii) admission in (tier, FCFS) order while the head of line fits; (iii) start the iteration.
     if (x.lane == 0) {
         const int n_decode = n;
-        long long prefill = 0;
+        int prefill = 0;
         int nr = n;
         while (nr < x.Bmax) {
             const uint32_t wm = x.wmask[i];
@@ -650,19 +694,20 @@ __device__ void form_batch(const Ctx &x, Cnt &cn, int i, long long base, long lo
             if (need > fr) break;
             const int k = __ffs(wm) - 1;
             const uint32_t r = pop_front(x, i, k, cn);
-            if (r == kNil) break;
+            if (r == kNone) break;
             const uint32_t P = x.plen[r], O = x.olen[r], gg = x.g[r];
-            st[nr] = s_make(P + gg, (uint32_t)need, O - gg, (uint32_t)k, gg == 0);
-            rd[nr] = r;
+            x.sst[i * x.BP + nr] = s_make(P + gg, (uint32_t)need, O - gg, (uint32_t)k, gg == 0);
+            x.srid[i * x.BP + nr] = r;
             ++nr;
             fr -= need;
-            prefill += (long long)(P + gg);
+            prefill += (int)(P + gg);
             refresh_hol(x, i);
         }
         x.nrun[i] = (uint8_t)nr;
         x.free_[i] = fr;
         if (nr > 0) {
-            const long long end = (long long)x.t + base + a_us * prefill + b_us * (long long)n_decode;
+            const long long end =
+                (long long)x.t + base + (long long)a_us * prefill + (long long)b_us * n_decode;
             if (end > 0xFFFFFFFELL) {
                 cn.status = SIM_ERR_OVERFLOW;
             } else {
@@ -676,14 +721,12 @@ __device__ void form_batch(const Ctx &x, Cnt &cn, int i, long long base, long lo
     __syncwarp();
 }
 
-__device__ __forceinline__ void copy_blob(unsigned char *dst, const unsigned char *src, uint32_t bytes, int lane) {
+__device__ __forceinline__ void copy16(unsigned char *dst, const unsigned char *src, uint32_t bytes, int lane) {
     for (uint32_t o = (uint32_t)lane * 16u; o < bytes; o += 512u)
         *reinterpret_cast<uint4 *>(dst + o) = *reinterpret_cast<const uint4 *>(src + o);
 }
 
-__device__ Ctx make_ctx(const Params &p, unsigned char *blob, int r, int lane) {
-    Ctx x;
-    const Layout &L = p.L;
+__device__ __forceinline__ void bind_blob(Ctx &x, const Layout &L, unsigned char *blob) {
     x.busy = reinterpret_cast<uint32_t *>(blob + L.busy);
     x.free_ = reinterpret_cast<int *>(blob + L.free_);
     x.resv = reinterpret_cast<int *>(blob + L.resv);
@@ -701,38 +744,23 @@ __device__ Ctx make_ctx(const Params &p, unsigned char *blob, int r, int lane) {
     x.head = reinterpret_cast<uint32_t *>(blob + L.head);
     x.tail = reinterpret_cast<uint32_t *>(blob + L.tail);
     x.h = reinterpret_cast<int *>(blob + L.h);
-    const long long o = p.offsets[r];
-    x.Q = (uint32_t)(p.offsets[r + 1] - o);
-    x.arrival = p.arrival + o;
-    x.plen = p.plen + o;
-    x.olen = p.olen + o;
-    x.tier = p.tier + o;
-    x.g = p.g + o;
-    x.link = p.link + o;
-    x.res = p.res + o;
-    x.srid = p.srid + (size_t)r * p.N * p.Bmax;
-    x.sst = p.sst + (size_t)r * p.N * p.Bmax;
-    x.log = p.log + (size_t)r * p.C;
-    x.N = p.N;
-    x.K = p.K;
-    x.M = p.M;
-    x.T = p.T;
-    x.tshift = p.tshift;
-    x.Bmax = p.Bmax;
-    x.S = p.S;
-    x.C = p.C;
-    x.c = p.c;
-    x.lane = lane;
-    x.t = 0;
-    return x;
 }
 
 // The persistent simulation kernel: each warp repeatedly takes a replica and
-// advances it by up to p.max_steps event times.
-__global__ void __launch_bounds__(64) k_run(Params p) {
+// advances it by up to p.max_steps event times.  C = instances per lane;
+// SMS = running-request slots staged in shared memory.
+template <int C, bool SMS>
+__global__ void __launch_bounds__(32 * kWarpsPerBlock) k_run(Params p) {
     extern __shared__ __align__(16) unsigned char smem[];
+    unsigned long long *magic = reinterpret_cast<unsigned long long *>(smem);
+    for (int d = threadIdx.x; d <= 64; d += blockDim.x)
+        magic[d] = d < 2 ? 0ull : ~0ull / (unsigned long long)d + 1ull;
+    __syncthreads();
     const int lane = threadIdx.x & 31;
-    unsigned char *blob = smem + (size_t)(threadIdx.x >> 5) * p.L.bytes;
+    const uint32_t per_warp = p.L.bytes + p.slot_bytes;
+    unsigned char *blob = smem + kMagicBytes + (size_t)(threadIdx.x >> 5) * per_warp;
+    unsigned char *sslots = blob + p.L.bytes;
+    const uint32_t nslot = p.NS;
     for (;;) {
         int r = 0;
         if (lane == 0) r = atomicAdd(p.work, 1);
@@ -741,9 +769,42 @@ __global__ void __launch_bounds__(64) k_run(Params p) {
         const RepState rs = p.rep[r];
         if (rs.status != SIM_REPLICA_RUNNING) continue;
         unsigned char *gblob = p.blobs + (size_t)r * p.L.bytes;
-        copy_blob(blob, gblob, p.L.bytes, lane);
+        uint64_t *g_sst = p.sst + (size_t)r * nslot;
+        uint32_t *g_srid = p.srid + (size_t)r * nslot;
+        copy16(blob, gblob, p.L.bytes, lane);
+        Ctx x;
+        bind_blob(x, p.L, blob);
+        if (SMS) {
+            x.sst = reinterpret_cast<uint64_t *>(sslots);
+            x.srid = reinterpret_cast<uint32_t *>(sslots + (size_t)nslot * 8);
+            copy16(sslots, reinterpret_cast<const unsigned char *>(g_sst), nslot * 8, lane);
+            copy16(sslots + (size_t)nslot * 8, reinterpret_cast<const unsigned char *>(g_srid), nslot * 4, lane);
+        } else {
+            x.sst = g_sst;
+            x.srid = g_srid;
+        }
         __syncwarp();
-        Ctx x = make_ctx(p, blob, r, lane);
+        const long long o = p.offsets[r];
+        x.Q = (uint32_t)(p.offsets[r + 1] - o);
+        x.arrival = p.arrival + o;
+        x.plen = p.plen + o;
+        x.olen = p.olen + o;
+        x.tier = p.tier + o;
+        x.g = p.g + o;
+        x.link = p.link + o;
+        x.res = p.res + o;
+        x.log = p.log + (size_t)r * p.cap;
+        x.magic = magic;
+        x.magT = p.magT;
+        x.N = p.N;
+        x.K = p.K;
+        x.T = p.T;
+        x.Bmax = p.Bmax;
+        x.BP = p.BP;
+        x.S = p.S;
+        x.cap = p.cap;
+        x.lane = lane;
+        x.t = rs.t;
         Cnt cn;
         cn.finished = rs.finished;
         cn.log_events = rs.log_events;
@@ -751,76 +812,78 @@ __global__ void __launch_bounds__(64) k_run(Params p) {
         cn.preemptions = rs.preemptions;
         cn.starts = rs.starts;
         cn.aborts = rs.aborts;
-        cn.steps = rs.steps;
-        cn.iterations = rs.iterations;
+        cn.steps = 0;
+        cn.iterations = 0;
         cn.member_iterations = rs.member_iterations;
         cn.events = rs.events;
         cn.status = SIM_REPLICA_RUNNING;
         uint32_t cursor = rs.cursor;
-        uint64_t next_tick = rs.next_tick;
-        uint64_t next_arr = cursor < x.Q ? (uint64_t)x.arrival[cursor] : kInf64;
-        x.t = rs.t;
-        long long here = 0;
+        uint32_t next_tick = rs.next_tick;
+        ArrBuf ab;
+        arr_refill(x, ab, cursor);
+        uint32_t next_arr = __shfl_sync(kFull, ab.time, 0);
+        const uint32_t max_steps = p.max_steps;
         for (;;) {
             if (cn.finished == x.Q) { cn.status = SIM_REPLICA_DONE; break; }
-            if (here >= p.max_steps) break;
+            if (cn.steps == max_steps) break;
             // a0: next event time
-            uint32_t mb = kIdle;
-            for (int j = 0; j < x.c; ++j) {
-                const int i = lane * x.c + j;
-                if (i < x.N) mb = min(mb, x.busy[i]);
+            uint32_t bz[C];
+            uint32_t mb = kNone;
+#pragma unroll
+            for (int j = 0; j < C; ++j) {
+                const int i = lane * C + j;
+                bz[j] = i < x.N ? x.busy[i] : kNone;
+                mb = min(mb, bz[j]);
             }
             const uint32_t tb = __reduce_min_sync(kFull, mb);
-            uint64_t tc = next_arr;
-            if (tb != kIdle && (uint64_t)tb < tc) tc = tb;
-            if (tc == kInf64) { cn.status = SIM_ERR_DEADLOCK; break; }
-            bool tick = false;
-            if (p.enable_mig && next_tick <= tc) { tc = next_tick; tick = true; }
-            x.t = (uint32_t)tc;
-            ++here;
+            const uint32_t tc = min(tb, next_arr);
+            if (tc == kNone) { cn.status = SIM_ERR_DEADLOCK; break; }
+            const bool tick = p.enable_mig && next_tick <= tc;
+            x.t = tick ? next_tick : tc;
             ++cn.steps;
             // 1. iteration ends, ascending instance index
             if (tb == x.t) {
                 uint32_t hits = 0;
-                for (int j = 0; j < x.c; ++j) {
-                    const int i = lane * x.c + j;
-                    if (i < x.N && x.busy[i] == x.t) hits |= 1u << j;
-                }
+#pragma unroll
+                for (int j = 0; j < C; ++j)
+                    if (bz[j] == x.t) hits |= 1u << j;
                 uint32_t lanes = __ballot_sync(kFull, hits != 0);
                 while (lanes) {
                     const int l = __ffs(lanes) - 1;
                     lanes &= lanes - 1;
-                    uint32_t h = __shfl_sync(kFull, hits, l);
+                    uint32_t h = C == 1 ? 1u : __shfl_sync(kFull, hits, l);
                     while (h) {
                         const int j = __ffs(h) - 1;
                         h &= h - 1;
-                        complete_instance(x, cn, l * x.c + j);
+                        complete_instance(x, cn, l * C + j);
                     }
                 }
             }
             // 2. dispatch of arrivals at t
-            if (next_arr == (uint64_t)x.t) dispatch_phase(x, cn, cursor, next_arr);
+            if (next_arr == x.t) dispatch_phase<C>(x, cn, cursor, next_arr, ab);
             // 3. migration tick
             if (tick) {
-                next_tick += p.interval;
-                migration_tick(x, cn, p.theta_num, p.theta_den);
+                const uint32_t nt = next_tick + p.interval;
+                next_tick = nt < next_tick ? kNone : nt;  // saturate: no tick beyond 2^32 - 1
+                migration_tick<C>(x, cn, p.theta_num, p.theta_den);
             }
             // 4. batch formation at idle instances with work, ascending index
             {
                 uint32_t want = 0;
-                for (int j = 0; j < x.c; ++j) {
-                    const int i = lane * x.c + j;
-                    if (i < x.N && x.busy[i] == kIdle && (x.nrun[i] > 0 || x.wmask[i] != 0)) want |= 1u << j;
+#pragma unroll
+                for (int j = 0; j < C; ++j) {
+                    const int i = lane * C + j;
+                    if (i < x.N && x.busy[i] == kNone && (x.nrun[i] | x.wmask[i]) != 0) want |= 1u << j;
                 }
                 uint32_t lanes = __ballot_sync(kFull, want != 0);
                 while (lanes) {
                     const int l = __ffs(lanes) - 1;
                     lanes &= lanes - 1;
-                    uint32_t h = __shfl_sync(kFull, want, l);
+                    uint32_t h = C == 1 ? 1u : __shfl_sync(kFull, want, l);
                     while (h) {
                         const int j = __ffs(h) - 1;
                         h &= h - 1;
-                        form_batch(x, cn, l * x.c + j, p.base, p.a, p.b);
+                        form_batch(x, cn, l * C + j, p.base, p.a, p.b);
                     }
                 }
             }
@@ -828,25 +891,30 @@ __global__ void __launch_bounds__(64) k_run(Params p) {
             if (cn.status < 0) break;
         }
         __syncwarp();
-        copy_blob(gblob, blob, p.L.bytes, lane);
+        copy16(gblob, blob, p.L.bytes, lane);
+        if (SMS) {
+            copy16(reinterpret_cast<unsigned char *>(g_sst), sslots, nslot * 8, lane);
+            copy16(reinterpret_cast<unsigned char *>(g_srid), sslots + (size_t)nslot * 8, nslot * 4, lane);
+        }
         if (lane == 0) {
-            RepState o;
-            o.t = x.t;
-            o.cursor = cursor;
-            o.finished = cn.finished;
-            o.log_events = cn.log_events;
-            o.next_tick = next_tick;
-            o.steps = cn.steps;
-            o.iterations = cn.iterations;
-            o.member_iterations = cn.member_iterations;
-            o.events = cn.events;
-            o.migrations = cn.migrations;
-            o.preemptions = cn.preemptions;
-            o.starts = cn.starts;
-            o.aborts = cn.aborts;
-            o.status = cn.status;
-            o.pad_[0] = o.pad_[1] = o.pad_[2] = 0;
-            p.rep[r] = o;
+            RepState o2;
+            o2.t = x.t;
+            o2.cursor = cursor;
+            o2.finished = cn.finished;
+            o2.log_events = cn.log_events;
+            o2.next_tick = next_tick;
+            o2.pad0 = 0;
+            o2.steps = rs.steps + cn.steps;
+            o2.iterations = rs.iterations + cn.iterations;
+            o2.member_iterations = cn.member_iterations;
+            o2.events = cn.events;
+            o2.migrations = cn.migrations;
+            o2.preemptions = cn.preemptions;
+            o2.starts = cn.starts;
+            o2.aborts = cn.aborts;
+            o2.status = cn.status;
+            o2.pad1 = 0;
+            p.rep[r] = o2;
         }
         __syncwarp();
     }
@@ -863,13 +931,13 @@ __global__ void k_init_state(Params p, const int *rep_table, const int *tbl_k, c
         const int tb = rep_table[r];
         const int K = tbl_k[tb];
         for (int i = lane; i < N; i += 32) {
-            reinterpret_cast<uint32_t *>(b + L.busy)[i] = kIdle;
+            reinterpret_cast<uint32_t *>(b + L.busy)[i] = kNone;
             reinterpret_cast<int *>(b + L.free_)[i] = p.M;
             reinterpret_cast<int *>(b + L.resv)[i] = 0;
             reinterpret_cast<int *>(b + L.hol)[i] = 0;
             reinterpret_cast<int *>(b + L.hr)[i] = 0;
             reinterpret_cast<int *>(b + L.key)[i] = 0;
-            reinterpret_cast<uint32_t *>(b + L.mreq)[i] = kNil;
+            reinterpret_cast<uint32_t *>(b + L.mreq)[i] = kNone;
             reinterpret_cast<int *>(b + L.mcopied)[i] = 0;
             reinterpret_cast<uint16_t *>(b + L.wmask)[i] = 0;
             b[L.nrun + i] = 0;
@@ -879,8 +947,8 @@ __global__ void k_init_state(Params p, const int *rep_table, const int *tbl_k, c
         }
         for (int i = lane; i < NK; i += 32) {
             reinterpret_cast<uint16_t *>(b + L.cnt)[i] = 0;
-            reinterpret_cast<uint32_t *>(b + L.head)[i] = kNil;
-            reinterpret_cast<uint32_t *>(b + L.tail)[i] = kNil;
+            reinterpret_cast<uint32_t *>(b + L.head)[i] = kNone;
+            reinterpret_cast<uint32_t *>(b + L.tail)[i] = kNone;
         }
         for (int k = lane; k < p.K; k += 32)
             reinterpret_cast<int *>(b + L.h)[k] = k < K ? tbl_h[tb * p.K + k] : 0;
@@ -896,7 +964,7 @@ __global__ void k_init_state(Params p, const int *rep_table, const int *tbl_k, c
 
 __global__ void k_init_requests(sim_request_result_t *res, uint16_t *g, long long n) {
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
-        reinterpret_cast<uint4 *>(res)[i] = make_uint4(0xFFFFFFFFu, kNil, kNil, 0u);
+        reinterpret_cast<uint4 *>(res)[i] = make_uint4(0xFFFFFFFFu, kNone, kNone, 0u);
         g[i] = 0;
     }
 }
@@ -916,7 +984,7 @@ __global__ void k_validate(const long long *offsets, int R, const uint32_t *arri
         if ((int)tier[i] >= tbl_k[rep_table[lo]]) f |= 2;
         if (plen[i] == 0 || olen[i] == 0) f |= 4;
         if ((long long)plen[i] + olen[i] > lim) f |= 8;
-        if (arrival[i] == kNil) f |= 16;
+        if (arrival[i] == kNone) f |= 16;
         if (f) atomicOr(flags, f);
     }
 }
@@ -944,6 +1012,84 @@ __global__ void k_export_stats(const RepState *rep, sim_replica_stats_t *out, in
     }
 }
 
+// ---- launch configuration ---------------------------------------------------
+typedef void (*RunKernel)(Params);
+
+template <bool SMS>
+RunKernel pick(int c) {
+    switch (c) {
+        case 1: return k_run<1, SMS>;
+        case 2: return k_run<2, SMS>;
+        case 4: return k_run<4, SMS>;
+        default: return k_run<8, SMS>;
+    }
+}
+
+struct Launch {
+    RunKernel fn = nullptr;
+    int grid = 0;
+    size_t smem = 0;
+    uint32_t slot_bytes = 0;
+};
+
+inline int lanes_c(int N) { return N <= 32 ? 1 : N <= 64 ? 2 : N <= 128 ? 4 : 8; }
+
+inline Layout make_layout(int N, int K) {
+    Layout L;
+    uint32_t o = 0;
+    auto take = [&](uint32_t bytes, uint32_t align) {
+        o = (o + align - 1) / align * align;
+        const uint32_t at = o;
+        o += bytes;
+        return at;
+    };
+    L.busy = take(4u * N, 16);
+    L.free_ = take(4u * N, 16);
+    L.resv = take(4u * N, 16);
+    L.hol = take(4u * N, 16);
+    L.hr = take(4u * N, 16);
+    L.key = take(4u * N, 16);
+    L.mreq = take(4u * N, 16);
+    L.mcopied = take(4u * N, 16);
+    L.head = take(4u * N * K, 16);
+    L.tail = take(4u * N * K, 16);
+    L.h = take(4u * K, 16);
+    L.wmask = take(2u * N, 16);
+    L.cnt = take(2u * N * K, 16);
+    L.nrun = take(N, 16);
+    L.nb = take(N, 16);
+    L.mrole = take(N, 16);
+    L.mpeer = take(N, 16);
+    L.bytes = (o + 15u) & ~15u;
+    return L;
+}
+
+// Chooses the kernel variant and grid for a problem; cudaSuccess or the error.
+inline uint32_t slots_per_replica(int N, int BP) { return ((uint32_t)N * (uint32_t)BP + 3u) & ~3u; }
+
+inline cudaError_t plan_launch(int R, int N, int BP, const Layout &L, Launch &out) {
+    const int c = lanes_c(N);
+    const uint32_t slots = slots_per_replica(N, BP) * 12u;
+    const bool sms = slots <= kSmemSlotLimit;
+    out.fn = sms ? pick<true>(c) : pick<false>(c);
+    out.slot_bytes = sms ? slots : 0u;
+    out.smem = kMagicBytes + (size_t)kWarpsPerBlock * (L.bytes + out.slot_bytes);
+    int dev = 0, sms_count = 0, per_sm = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms_count, cudaDevAttrMultiProcessorCount, dev);
+    if (e == cudaSuccess && out.smem > 48 * 1024)
+        e = cudaFuncSetAttribute(out.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)out.smem);
+    if (e == cudaSuccess)
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, out.fn, 32 * kWarpsPerBlock, out.smem);
+    if (e != cudaSuccess) return e;
+    if (per_sm < 1) return cudaErrorInvalidConfiguration;
+    const long long want = ((long long)R + kWarpsPerBlock - 1) / kWarpsPerBlock;
+    out.grid = (int)std::min<long long>(want, (long long)sms_count * per_sm);
+    return cudaSuccess;
+}
+
+inline unsigned long long magic40(unsigned d) { return ((1ull << kMagicShift) + d - 1ull) / d; }
+
 }  // namespace mt
 
 // ============================================================================
@@ -952,12 +1098,13 @@ __global__ void k_export_stats(const RepState *rep, sim_replica_stats_t *out, in
 struct sim {
     sim_cluster_t cl;
     sim_policy_t pol;
-    int K = 0, ntables = 0, c = 1, tshift = -1;
+    int K = 0, ntables = 0, BP = 0;
     std::vector<int> tbl_k, tbl_h, rep_table;
     cudaStream_t stream = nullptr;
     sim_allocator_t al{};
     bool use_al = false;
     mt::Layout L{};
+    mt::Launch launch{};
     struct Buf { void *p; size_t n; };
     std::vector<Buf> bufs;
     size_t dev_bytes = 0;
@@ -977,8 +1124,7 @@ struct sim {
     uint8_t *d_tier = nullptr;
     uint2 *d_link = nullptr;
     sim_request_result_t *d_res = nullptr;
-    int sms = 0, grid = 0, wpb = 2;
-    size_t smem = 0;
+    int sms = 0;
     std::string err;
 };
 
@@ -1030,57 +1176,36 @@ void dfree(sim_t *s, void *p) {
     }
 }
 
-mt::Layout make_layout(int N, int K) {
-    mt::Layout L;
-    uint32_t o = 0;
-    auto take = [&](uint32_t bytes, uint32_t align) {
-        o = (o + align - 1) / align * align;
-        const uint32_t at = o;
-        o += bytes;
-        return at;
-    };
-    L.busy = take(4u * N, 16);
-    L.free_ = take(4u * N, 16);
-    L.resv = take(4u * N, 16);
-    L.hol = take(4u * N, 16);
-    L.hr = take(4u * N, 16);
-    L.key = take(4u * N, 16);
-    L.mreq = take(4u * N, 16);
-    L.mcopied = take(4u * N, 16);
-    L.head = take(4u * N * K, 16);
-    L.tail = take(4u * N * K, 16);
-    L.h = take(4u * K, 16);
-    L.wmask = take(2u * N, 16);
-    L.cnt = take(2u * N * K, 16);
-    L.nrun = take(N, 16);
-    L.nb = take(N, 16);
-    L.mrole = take(N, 16);
-    L.mpeer = take(N, 16);
-    L.bytes = (o + 15u) & ~15u;
-    return L;
+// Fills the scalar part of the kernel parameters (pointers are set by the caller).
+void fill_scalars(mt::Params &p, const sim_cluster_t &cl, const sim_policy_t &pol, int K, int cap,
+                  const mt::Layout &L, uint32_t slot_bytes, long long max_steps) {
+    p.R = cl.num_replicas;
+    p.N = cl.num_instances;
+    p.M = cl.blocks_per_instance;
+    p.T = cl.tokens_per_block;
+    p.Bmax = cl.max_batch;
+    p.BP = (cl.max_batch + 1) & ~1;
+    p.NS = mt::slots_per_replica(cl.num_instances, p.BP);
+    p.K = K;
+    p.S = pol.migrate_blocks_per_iter;
+    p.cap = cap;
+    p.enable_mig = pol.enable_migration;
+    p.theta_num = pol.theta_num;
+    p.theta_den = pol.theta_den;
+    p.interval = (uint32_t)pol.migrate_interval_us;
+    p.max_steps = (uint32_t)std::min<long long>(max_steps, 0xFFFFFFFFLL);
+    p.magT = mt::magic40((unsigned)cl.tokens_per_block);
+    p.base = (int)pol.iter_base_us;
+    p.a = (int)pol.iter_us_per_prefill_token;
+    p.b = (int)pol.iter_us_per_decode_seq;
+    p.L = L;
+    p.slot_bytes = slot_bytes;
 }
 
 mt::Params make_params(const sim_t *s, long long max_steps) {
     mt::Params p;
-    p.R = s->cl.num_replicas;
-    p.N = s->cl.num_instances;
-    p.M = s->cl.blocks_per_instance;
-    p.T = s->cl.tokens_per_block;
-    p.tshift = s->tshift;
-    p.Bmax = s->cl.max_batch;
-    p.K = s->K;
-    p.c = s->c;
-    p.S = s->pol.migrate_blocks_per_iter;
-    p.C = s->pol.event_log_capacity;
-    p.enable_mig = s->pol.enable_migration;
-    p.theta_num = s->pol.theta_num;
-    p.theta_den = s->pol.theta_den;
-    p.interval = (uint32_t)s->pol.migrate_interval_us;
-    p.base = s->pol.iter_base_us;
-    p.a = s->pol.iter_us_per_prefill_token;
-    p.b = s->pol.iter_us_per_decode_seq;
-    p.max_steps = max_steps;
-    p.L = s->L;
+    memset(&p, 0, sizeof p);
+    fill_scalars(p, s->cl, s->pol, s->K, s->pol.event_log_capacity, s->L, s->launch.slot_bytes, max_steps);
     p.offsets = s->d_off;
     p.arrival = s->d_arrival;
     p.plen = s->d_plen;
@@ -1107,8 +1232,7 @@ int check_launch(sim_t *s, const char *what) {
 int reset_state(sim_t *s) {
     mt::Params p = make_params(s, 0);
     const int R = s->cl.num_replicas;
-    const int blocks = (R + 7) / 8;
-    mt::k_init_state<<<blocks, 256, 0, s->stream>>>(p, s->d_rep_table, s->d_tbl_k, s->d_tbl_h);
+    mt::k_init_state<<<(R + 7) / 8, 256, 0, s->stream>>>(p, s->d_rep_table, s->d_tbl_k, s->d_tbl_h);
     int rc = check_launch(s, "k_init_state");
     if (rc) return rc;
     if (s->qtot > 0) {
@@ -1117,6 +1241,55 @@ int reset_state(sim_t *s) {
         rc = check_launch(s, "k_init_requests");
     }
     return rc;
+}
+
+// The limits every entry point enforces on cluster, tier tables and policy.
+int validate_config(sim_t *s, const sim_cluster_t *cl, const sim_tier_table_t *tt, const sim_policy_t *pol) {
+    if (!cl || !tt || !pol) return fail(s, SIM_ERR_ARG, "cluster, tiers and policy are required");
+    if (cl->num_replicas < 1) return fail(s, SIM_ERR_ARG, "num_replicas must be >= 1");
+    if (cl->num_instances < 1 || cl->num_instances > SIM_MAX_INSTANCES)
+        return fail(s, SIM_ERR_ARG, "num_instances must be in [1, %d]", SIM_MAX_INSTANCES);
+    if (cl->blocks_per_instance < 1 || cl->blocks_per_instance > SIM_MAX_BLOCKS)
+        return fail(s, SIM_ERR_ARG, "blocks_per_instance must be in [1, %d]", SIM_MAX_BLOCKS);
+    if (cl->tokens_per_block < 1 || cl->tokens_per_block > 65535)
+        return fail(s, SIM_ERR_ARG, "tokens_per_block must be in [1, 65535]");
+    if (cl->max_batch < 1 || cl->max_batch > SIM_MAX_BATCH)
+        return fail(s, SIM_ERR_ARG, "max_batch must be in [1, %d]", SIM_MAX_BATCH);
+    if (tt->num_tables < 1 || tt->max_tiers < 1 || tt->max_tiers > SIM_MAX_TIERS)
+        return fail(s, SIM_ERR_ARG, "need num_tables >= 1 and max_tiers in [1, %d]", SIM_MAX_TIERS);
+    if (!tt->num_tiers || !tt->headroom_blocks || !tt->replica_table)
+        return fail(s, SIM_ERR_ARG, "tier table pointers must not be NULL");
+    for (int t = 0; t < tt->num_tables; ++t) {
+        const int K = tt->num_tiers[t];
+        if (K < 1 || K > tt->max_tiers) return fail(s, SIM_ERR_ARG, "table %d: num_tiers out of range", t);
+        long long sum = 0;
+        for (int k = 0; k < K; ++k) {
+            const int h = tt->headroom_blocks[t * tt->max_tiers + k];
+            if (h < 0) return fail(s, SIM_ERR_ARG, "table %d: negative headroom", t);
+            sum += h;
+        }
+        if (cl->blocks_per_instance + sum >= mt::kMaxKeyRange)
+            return fail(s, SIM_ERR_ARG, "table %d: M + sum of headroom must be below 2^19", t);
+    }
+    for (int r = 0; r < cl->num_replicas; ++r)
+        if (tt->replica_table[r] < 0 || tt->replica_table[r] >= tt->num_tables)
+            return fail(s, SIM_ERR_ARG, "replica %d: table index out of range", r);
+    if (pol->policy != SIM_POLICY_LLUMNIX_MT) return fail(s, SIM_ERR_ARG, "unknown policy %d", pol->policy);
+    if (pol->enable_migration != 0 && pol->enable_migration != 1)
+        return fail(s, SIM_ERR_ARG, "enable_migration must be 0 or 1");
+    const long long lim24 = 1LL << 24;
+    if (pol->iter_base_us < 0 || pol->iter_base_us > lim24 || pol->iter_us_per_prefill_token < 0 ||
+        pol->iter_us_per_prefill_token > lim24 || pol->iter_us_per_decode_seq < 0 || pol->iter_us_per_decode_seq > lim24)
+        return fail(s, SIM_ERR_ARG, "iteration-time coefficients must be in [0, 2^24]");
+    if (pol->migrate_blocks_per_iter < 1 || pol->migrate_blocks_per_iter > 65535)
+        return fail(s, SIM_ERR_ARG, "migrate_blocks_per_iter must be in [1, 65535]");
+    if (pol->theta_den < 1 || pol->theta_num < 0 || pol->theta_num > (1 << 20) || pol->theta_den > (1 << 20))
+        return fail(s, SIM_ERR_ARG, "theta must be num/den with num in [0, 2^20], den in [1, 2^20]");
+    if (pol->event_log_capacity < 0 || pol->event_log_capacity > (1 << 24))
+        return fail(s, SIM_ERR_ARG, "event_log_capacity must be in [0, 2^24]");
+    if (pol->migrate_interval_us < 1 || pol->migrate_interval_us > (1LL << 31))
+        return fail(s, SIM_ERR_ARG, "migrate_interval_us must be in [1, 2^31]");
+    return SIM_OK;
 }
 
 }  // namespace
@@ -1146,50 +1319,8 @@ int sim_create(const sim_cluster_t *cl, const sim_tier_table_t *tt, const sim_po
                const sim_allocator_t *allocator, sim_t **out) {
     if (!out) return fail(nullptr, SIM_ERR_ARG, "out is NULL");
     *out = nullptr;
-    if (!cl || !tt || !pol) return fail(nullptr, SIM_ERR_ARG, "cluster, tiers and policy are required");
-    if (cl->num_replicas < 1) return fail(nullptr, SIM_ERR_ARG, "num_replicas must be >= 1");
-    if (cl->num_instances < 1 || cl->num_instances > SIM_MAX_INSTANCES)
-        return fail(nullptr, SIM_ERR_ARG, "num_instances must be in [1, %d]", SIM_MAX_INSTANCES);
-    if (cl->blocks_per_instance < 1 || cl->blocks_per_instance > SIM_MAX_BLOCKS)
-        return fail(nullptr, SIM_ERR_ARG, "blocks_per_instance must be in [1, %d]", SIM_MAX_BLOCKS);
-    if (cl->tokens_per_block < 1 || cl->tokens_per_block > 65535)
-        return fail(nullptr, SIM_ERR_ARG, "tokens_per_block must be in [1, 65535]");
-    if (cl->max_batch < 1 || cl->max_batch > SIM_MAX_BATCH)
-        return fail(nullptr, SIM_ERR_ARG, "max_batch must be in [1, %d]", SIM_MAX_BATCH);
-    if (tt->num_tables < 1 || tt->max_tiers < 1 || tt->max_tiers > SIM_MAX_TIERS)
-        return fail(nullptr, SIM_ERR_ARG, "need num_tables >= 1 and max_tiers in [1, %d]", SIM_MAX_TIERS);
-    if (!tt->num_tiers || !tt->headroom_blocks || !tt->replica_table)
-        return fail(nullptr, SIM_ERR_ARG, "tier table pointers must not be NULL");
-    for (int t = 0; t < tt->num_tables; ++t) {
-        const int K = tt->num_tiers[t];
-        if (K < 1 || K > tt->max_tiers) return fail(nullptr, SIM_ERR_ARG, "table %d: num_tiers out of range", t);
-        long long sum = 0;
-        for (int k = 0; k < K; ++k) {
-            const int h = tt->headroom_blocks[t * tt->max_tiers + k];
-            if (h < 0) return fail(nullptr, SIM_ERR_ARG, "table %d: negative headroom", t);
-            sum += h;
-        }
-        if (cl->blocks_per_instance + sum >= mt::kMaxKeyRange)
-            return fail(nullptr, SIM_ERR_ARG, "table %d: M + sum of headroom must be below 2^19", t);
-    }
-    for (int r = 0; r < cl->num_replicas; ++r)
-        if (tt->replica_table[r] < 0 || tt->replica_table[r] >= tt->num_tables)
-            return fail(nullptr, SIM_ERR_ARG, "replica %d: table index out of range", r);
-    if (pol->policy != SIM_POLICY_LLUMNIX_MT) return fail(nullptr, SIM_ERR_ARG, "unknown policy %d", pol->policy);
-    if (pol->enable_migration != 0 && pol->enable_migration != 1)
-        return fail(nullptr, SIM_ERR_ARG, "enable_migration must be 0 or 1");
-    const long long lim24 = 1LL << 24;
-    if (pol->iter_base_us < 0 || pol->iter_base_us > lim24 || pol->iter_us_per_prefill_token < 0 ||
-        pol->iter_us_per_prefill_token > lim24 || pol->iter_us_per_decode_seq < 0 || pol->iter_us_per_decode_seq > lim24)
-        return fail(nullptr, SIM_ERR_ARG, "iteration-time coefficients must be in [0, 2^24]");
-    if (pol->migrate_blocks_per_iter < 1 || pol->migrate_blocks_per_iter > 65535)
-        return fail(nullptr, SIM_ERR_ARG, "migrate_blocks_per_iter must be in [1, 65535]");
-    if (pol->theta_den < 1 || pol->theta_num < 0 || pol->theta_num > (1 << 20) || pol->theta_den > (1 << 20))
-        return fail(nullptr, SIM_ERR_ARG, "theta must be num/den with num in [0, 2^20], den in [1, 2^20]");
-    if (pol->event_log_capacity < 0 || pol->event_log_capacity > (1 << 24))
-        return fail(nullptr, SIM_ERR_ARG, "event_log_capacity must be in [0, 2^24]");
-    if (pol->migrate_interval_us < 1 || pol->migrate_interval_us > (1LL << 31))
-        return fail(nullptr, SIM_ERR_ARG, "migrate_interval_us must be in [1, 2^31]");
+    int rc = validate_config(nullptr, cl, tt, pol);
+    if (rc) return rc;
     if (allocator && (!allocator->alloc || !allocator->free))
         return fail(nullptr, SIM_ERR_ARG, "allocator needs both alloc and free");
 
@@ -1199,23 +1330,21 @@ int sim_create(const sim_cluster_t *cl, const sim_tier_table_t *tt, const sim_po
     s->pol = *pol;
     s->K = tt->max_tiers;
     s->ntables = tt->num_tables;
+    s->BP = (cl->max_batch + 1) & ~1;
     s->tbl_k.assign(tt->num_tiers, tt->num_tiers + tt->num_tables);
     s->tbl_h.assign(tt->headroom_blocks, tt->headroom_blocks + (size_t)tt->num_tables * tt->max_tiers);
     s->rep_table.assign(tt->replica_table, tt->replica_table + cl->num_replicas);
     s->stream = (cudaStream_t)cuda_stream;
     if (allocator) { s->al = *allocator; s->use_al = true; }
-    s->c = (cl->num_instances + 31) / 32;
-    const int T = cl->tokens_per_block;
-    s->tshift = (T & (T - 1)) == 0 ? __builtin_ctz((unsigned)T) : -1;
-    s->L = make_layout(cl->num_instances, s->K);
+    s->L = mt::make_layout(cl->num_instances, s->K);
 
-    const size_t R = (size_t)cl->num_replicas, N = (size_t)cl->num_instances, B = (size_t)cl->max_batch;
+    const size_t R = (size_t)cl->num_replicas, NS = mt::slots_per_replica(cl->num_instances, s->BP);
     s->d_rep_table = (int *)dalloc(s, R * 4);
     s->d_tbl_k = (int *)dalloc(s, (size_t)s->ntables * 4);
     s->d_tbl_h = (int *)dalloc(s, (size_t)s->ntables * s->K * 4);
     s->d_blobs = (unsigned char *)dalloc(s, R * s->L.bytes);
-    s->d_srid = (uint32_t *)dalloc(s, R * N * B * 4);
-    s->d_sst = (uint64_t *)dalloc(s, R * N * B * 8);
+    s->d_srid = (uint32_t *)dalloc(s, R * NS * 4);
+    s->d_sst = (uint64_t *)dalloc(s, R * NS * 8);
     s->d_rep = (mt::RepState *)dalloc(s, R * sizeof(mt::RepState));
     s->d_log = (sim_migration_event_t *)dalloc(s, R * (size_t)pol->event_log_capacity * sizeof(sim_migration_event_t));
     s->d_work = (int *)dalloc(s, 16);
@@ -1234,24 +1363,15 @@ int sim_create(const sim_cluster_t *cl, const sim_tier_table_t *tt, const sim_po
     int dev = 0;
     if (e == cudaSuccess) e = cudaGetDevice(&dev);
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&s->sms, cudaDevAttrMultiProcessorCount, dev);
-    s->smem = (size_t)s->wpb * s->L.bytes;
-    if (e == cudaSuccess && s->smem > 48 * 1024)
-        e = cudaFuncSetAttribute(mt::k_run, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)s->smem);
-    int per_sm = 0;
-    if (e == cudaSuccess)
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, mt::k_run, 32 * s->wpb, s->smem);
+    if (e == cudaSuccess) e = mt::plan_launch(cl->num_replicas, cl->num_instances, s->BP, s->L, s->launch);
     if (e != cudaSuccess) {
         cudaGetLastError();
-        int rc = cuda_fail(nullptr, e, "sim_create");
+        rc = e == cudaErrorInvalidConfiguration
+                 ? fail(nullptr, SIM_ERR_ARG, "per-replica state (%u bytes) does not fit in shared memory", s->L.bytes)
+                 : cuda_fail(nullptr, e, "sim_create");
         sim_destroy(s);
         return rc;
     }
-    if (per_sm < 1) {
-        sim_destroy(s);
-        return fail(nullptr, SIM_ERR_ARG, "per-replica state (%u bytes) does not fit in shared memory", s->L.bytes);
-    }
-    const long long want = ((long long)R + s->wpb - 1) / s->wpb;
-    s->grid = (int)std::min<long long>(want, (long long)s->sms * per_sm);
     *out = s;
     return SIM_OK;
 }
@@ -1342,7 +1462,7 @@ int sim_run(sim_t *s, int64_t max_steps, int64_t *num_unfinished) {
     cudaError_t e = cudaMemsetAsync(s->d_work, 0, 4, s->stream);
     if (e != cudaSuccess) return cuda_fail(s, e, "sim_run");
     mt::Params p = make_params(s, (long long)max_steps);
-    mt::k_run<<<s->grid, 32 * s->wpb, s->smem, s->stream>>>(p);
+    s->launch.fn<<<s->launch.grid, 32 * mt::kWarpsPerBlock, s->launch.smem, s->stream>>>(p);
     int rc = check_launch(s, "k_run");
     if (rc) return rc;
     if (num_unfinished) {
@@ -1418,53 +1538,6 @@ namespace {
 constexpr int kMaxDevices = 64;
 void *g_static_scratch_addr[kMaxDevices];  // device address of g_static_scratch, looked up once per device
 
-int static_fail(int code, const char *fmt, ...) {
-    char buf[512];
-    va_list ap;
-    va_start(ap, fmt);
-    vsnprintf(buf, sizeof buf, fmt, ap);
-    va_end(ap);
-    g_create_err = buf;
-    return code;
-}
-
-// The same limits sim_create enforces.
-int static_validate(const sim_cluster_t *cl, const sim_tier_table_t *tt, const sim_policy_t *pol) {
-    if (!cl || !tt || !pol) return static_fail(SIM_ERR_ARG, "cluster, tiers and policy are required");
-    if (cl->num_replicas < 1 || cl->num_instances < 1 || cl->num_instances > SIM_MAX_INSTANCES ||
-        cl->blocks_per_instance < 1 || cl->blocks_per_instance > SIM_MAX_BLOCKS || cl->tokens_per_block < 1 ||
-        cl->tokens_per_block > 65535 || cl->max_batch < 1 || cl->max_batch > SIM_MAX_BATCH)
-        return static_fail(SIM_ERR_ARG, "cluster shape out of range");
-    if (tt->num_tables < 1 || tt->max_tiers < 1 || tt->max_tiers > SIM_MAX_TIERS || !tt->num_tiers ||
-        !tt->headroom_blocks || !tt->replica_table)
-        return static_fail(SIM_ERR_ARG, "invalid tier tables");
-    for (int t = 0; t < tt->num_tables; ++t) {
-        const int K = tt->num_tiers[t];
-        if (K < 1 || K > tt->max_tiers) return static_fail(SIM_ERR_ARG, "table %d: num_tiers out of range", t);
-        long long sum = 0;
-        for (int k = 0; k < K; ++k) {
-            const int h = tt->headroom_blocks[t * tt->max_tiers + k];
-            if (h < 0) return static_fail(SIM_ERR_ARG, "table %d: negative headroom", t);
-            sum += h;
-        }
-        if (cl->blocks_per_instance + sum >= mt::kMaxKeyRange)
-            return static_fail(SIM_ERR_ARG, "table %d: M + sum of headroom must be below 2^19", t);
-    }
-    for (int r = 0; r < cl->num_replicas; ++r)
-        if (tt->replica_table[r] < 0 || tt->replica_table[r] >= tt->num_tables)
-            return static_fail(SIM_ERR_ARG, "replica %d: table index out of range", r);
-    const long long lim24 = 1LL << 24;
-    if (pol->policy != SIM_POLICY_LLUMNIX_MT || (pol->enable_migration != 0 && pol->enable_migration != 1) ||
-        pol->iter_base_us < 0 || pol->iter_base_us > lim24 || pol->iter_us_per_prefill_token < 0 ||
-        pol->iter_us_per_prefill_token > lim24 || pol->iter_us_per_decode_seq < 0 ||
-        pol->iter_us_per_decode_seq > lim24 || pol->migrate_blocks_per_iter < 1 ||
-        pol->migrate_blocks_per_iter > 65535 || pol->theta_den < 1 || pol->theta_num < 0 ||
-        pol->theta_num > (1 << 20) || pol->theta_den > (1 << 20) || pol->event_log_capacity < 0 ||
-        pol->event_log_capacity > (1 << 24) || pol->migrate_interval_us < 1 || pol->migrate_interval_us > (1LL << 31))
-        return static_fail(SIM_ERR_ARG, "policy out of range");
-    return SIM_OK;
-}
-
 size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 }  // namespace
@@ -1473,29 +1546,30 @@ extern "C" int sim_run_static(const sim_cluster_t *cl, const sim_tier_table_t *t
                               const int64_t *off, const uint32_t *arrival, const uint16_t *plen,
                               const uint16_t *olen, const uint8_t *tier, sim_request_result_t *per_request,
                               sim_replica_stats_t *per_replica, sim_migration_event_t *events, void *cuda_stream) {
-    int rc = static_validate(cl, tt, pol);
+    int rc = validate_config(nullptr, cl, tt, pol);
     if (rc) return rc;
-    if (!off) return static_fail(SIM_ERR_ARG, "replica_offsets is NULL");
+    if (!off) return fail(nullptr, SIM_ERR_ARG, "replica_offsets is NULL");
     const int R = cl->num_replicas;
-    if (off[0] != 0) return static_fail(SIM_ERR_TRACE, "replica_offsets[0] must be 0");
+    if (off[0] != 0) return fail(nullptr, SIM_ERR_TRACE, "replica_offsets[0] must be 0");
     for (int r = 0; r < R; ++r) {
         const int64_t q = off[r + 1] - off[r];
         if (q < 0 || q > (int64_t)0xFFFFFFFEll)
-            return static_fail(SIM_ERR_TRACE, "replica_offsets invalid at replica %d", r);
+            return fail(nullptr, SIM_ERR_TRACE, "replica_offsets invalid at replica %d", r);
     }
     const int64_t n = off[R];
     if (n > 0 && (!arrival || !plen || !olen || !tier || !per_request))
-        return static_fail(SIM_ERR_ARG, "trace and per_request pointers must not be NULL");
-    if (!per_replica) return static_fail(SIM_ERR_ARG, "per_replica must not be NULL");
+        return fail(nullptr, SIM_ERR_ARG, "trace and per_request pointers must not be NULL");
+    if (!per_replica) return fail(nullptr, SIM_ERR_ARG, "per_replica must not be NULL");
     const int cap = events ? pol->event_log_capacity : 0;
 
     // Carve the scratch array.
-    const int N = cl->num_instances, B = cl->max_batch, K = tt->max_tiers;
-    const mt::Layout L = make_layout(N, K);
+    const int N = cl->num_instances, BP = (cl->max_batch + 1) & ~1, K = tt->max_tiers;
+    const mt::Layout L = mt::make_layout(N, K);
     size_t o = 0;
     const size_t o_blobs = o; o = align256(o + (size_t)R * L.bytes);
-    const size_t o_srid = o; o = align256(o + (size_t)R * N * B * 4);
-    const size_t o_sst = o; o = align256(o + (size_t)R * N * B * 8);
+    const size_t NS = mt::slots_per_replica(N, BP);
+    const size_t o_srid = o; o = align256(o + (size_t)R * NS * 4);
+    const size_t o_sst = o; o = align256(o + (size_t)R * NS * 8);
     const size_t o_rep = o; o = align256(o + (size_t)R * sizeof(mt::RepState));
     const size_t o_g = o; o = align256(o + (size_t)n * 2);
     const size_t o_link = o; o = align256(o + (size_t)n * 8);
@@ -1505,44 +1579,34 @@ extern "C" int sim_run_static(const sim_cluster_t *cl, const sim_tier_table_t *t
     const size_t o_th = o; o = align256(o + (size_t)tt->num_tables * K * 4);
     const size_t o_work = o; o = align256(o + 16);
     if (o > (size_t)SIM_STATIC_SCRATCH_BYTES)
-        return static_fail(SIM_ERR_ARG, "problem needs %zu bytes of scratch; sim_run_static holds %u bytes", o,
-                           (unsigned)SIM_STATIC_SCRATCH_BYTES);
+        return fail(nullptr, SIM_ERR_ARG, "problem needs %zu bytes of scratch; sim_run_static holds %u bytes", o,
+                    (unsigned)SIM_STATIC_SCRATCH_BYTES);
 
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return static_fail(SIM_ERR_CUDA, "cudaGetDevice: %s", cudaGetErrorString(e));
-    if (dev < 0 || dev >= kMaxDevices) return static_fail(SIM_ERR_ARG, "device index %d not supported", dev);
+    if (e != cudaSuccess) return fail(nullptr, SIM_ERR_CUDA, "cudaGetDevice: %s", cudaGetErrorString(e));
+    if (dev < 0 || dev >= kMaxDevices) return fail(nullptr, SIM_ERR_ARG, "device index %d not supported", dev);
     if (!g_static_scratch_addr[dev]) {
         void *p = nullptr;
         e = cudaGetSymbolAddress(&p, g_static_scratch);
         if (e != cudaSuccess || !p)
-            return static_fail(SIM_ERR_CUDA, "cudaGetSymbolAddress: %s", cudaGetErrorString(e));
+            return fail(nullptr, SIM_ERR_CUDA, "cudaGetSymbolAddress: %s", cudaGetErrorString(e));
         g_static_scratch_addr[dev] = p;
     }
     unsigned char *base = (unsigned char *)g_static_scratch_addr[dev];
     cudaStream_t st = (cudaStream_t)cuda_stream;
 
+    mt::Launch lc;
+    e = mt::plan_launch(R, N, BP, L, lc);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return e == cudaErrorInvalidConfiguration
+                   ? fail(nullptr, SIM_ERR_ARG, "per-replica state does not fit in shared memory")
+                   : fail(nullptr, SIM_ERR_CUDA, "sim_run_static launch set-up: %s", cudaGetErrorString(e));
+    }
     mt::Params p;
     memset(&p, 0, sizeof p);
-    p.R = R;
-    p.N = N;
-    p.M = cl->blocks_per_instance;
-    p.T = cl->tokens_per_block;
-    p.tshift = (p.T & (p.T - 1)) == 0 ? __builtin_ctz((unsigned)p.T) : -1;
-    p.Bmax = B;
-    p.K = K;
-    p.c = (N + 31) / 32;
-    p.S = pol->migrate_blocks_per_iter;
-    p.C = cap;
-    p.enable_mig = pol->enable_migration;
-    p.theta_num = pol->theta_num;
-    p.theta_den = pol->theta_den;
-    p.interval = (uint32_t)pol->migrate_interval_us;
-    p.base = pol->iter_base_us;
-    p.a = pol->iter_us_per_prefill_token;
-    p.b = pol->iter_us_per_decode_seq;
-    p.max_steps = 1LL << 62;
-    p.L = L;
+    fill_scalars(p, *cl, *pol, K, cap, L, lc.slot_bytes, 1LL << 62);
     p.offsets = (const long long *)(base + o_off);
     p.arrival = arrival;
     p.plen = plen;
@@ -1566,10 +1630,10 @@ extern "C" int sim_run_static(const sim_cluster_t *cl, const sim_tier_table_t *t
     if (e == cudaSuccess)
         e = cudaMemcpyAsync(th, tt->headroom_blocks, (size_t)tt->num_tables * K * 4, cudaMemcpyHostToDevice, st);
     if (e == cudaSuccess) e = cudaMemsetAsync(p.work, 0, 16, st);
-    if (e != cudaSuccess) return static_fail(SIM_ERR_CUDA, "sim_run_static copy: %s", cudaGetErrorString(e));
+    if (e != cudaSuccess) return fail(nullptr, SIM_ERR_CUDA, "sim_run_static copy: %s", cudaGetErrorString(e));
     int sms = 0;
     e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    if (e != cudaSuccess) return static_fail(SIM_ERR_CUDA, "sim_run_static: %s", cudaGetErrorString(e));
+    if (e != cudaSuccess) return fail(nullptr, SIM_ERR_CUDA, "sim_run_static: %s", cudaGetErrorString(e));
     if (n > 0) {
         const long long lim = std::min<long long>((long long)p.M * p.T, 65536);
         const long long nb = std::min<long long>((n + 255) / 256, (long long)sms * 32);
@@ -1579,28 +1643,19 @@ extern "C" int sim_run_static(const sim_cluster_t *cl, const sim_tier_table_t *t
         e = cudaGetLastError();
         if (e == cudaSuccess) e = cudaMemcpyAsync(&flags, p.work + 1, 4, cudaMemcpyDeviceToHost, st);
         if (e == cudaSuccess) e = cudaStreamSynchronize(st);
-        if (e != cudaSuccess) return static_fail(SIM_ERR_CUDA, "sim_run_static validation: %s", cudaGetErrorString(e));
-        if (flags) return static_fail(SIM_ERR_TRACE, "malformed trace (validation flags 0x%x)", flags);
+        if (e != cudaSuccess)
+            return fail(nullptr, SIM_ERR_CUDA, "sim_run_static validation: %s", cudaGetErrorString(e));
+        if (flags) return fail(nullptr, SIM_ERR_TRACE, "malformed trace (validation flags 0x%x)", flags);
     }
     mt::k_init_state<<<(R + 7) / 8, 256, 0, st>>>(p, rt, tk, th);
     if (n > 0) {
         const long long nb = std::min<long long>((n + 255) / 256, 65535LL * 16);
         mt::k_init_requests<<<(unsigned)nb, 256, 0, st>>>(per_request, p.g, (long long)n);
     }
-    const int wpb = 2;
-    const size_t smem = (size_t)wpb * L.bytes;
-    e = cudaGetLastError();
-    if (e == cudaSuccess && smem > 48 * 1024)
-        e = cudaFuncSetAttribute(mt::k_run, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    int per_sm = 0;
-    if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, mt::k_run, 32 * wpb, smem);
-    if (e != cudaSuccess) return static_fail(SIM_ERR_CUDA, "sim_run_static launch set-up: %s", cudaGetErrorString(e));
-    if (per_sm < 1) return static_fail(SIM_ERR_ARG, "per-replica state does not fit in shared memory");
-    const int grid = (int)std::min<long long>(((long long)R + wpb - 1) / wpb, (long long)sms * per_sm);
-    mt::k_run<<<grid, 32 * wpb, smem, st>>>(p);
+    lc.fn<<<lc.grid, 32 * mt::kWarpsPerBlock, lc.smem, st>>>(p);
     mt::k_export_stats<<<(R + 255) / 256, 256, 0, st>>>(p.rep, per_replica, R, nullptr);
     e = cudaGetLastError();
     if (e == cudaSuccess) e = cudaStreamSynchronize(st);
-    if (e != cudaSuccess) return static_fail(SIM_ERR_CUDA, "sim_run_static: %s", cudaGetErrorString(e));
+    if (e != cudaSuccess) return fail(nullptr, SIM_ERR_CUDA, "sim_run_static: %s", cudaGetErrorString(e));
     return SIM_OK;
 }
