@@ -62,8 +62,9 @@ constexpr int kKeyShift = 12;            // keys are floor(num * 4096 / den)
 constexpr int kMaxKeyRange = 1 << 19;    // |num| < 2^19 keeps num * 4096 below 2^31
 constexpr int kMagicShift = 40;          // floor(n / T) = (n * ceil(2^40 / T)) >> 40 for n < 2^20, T <= 65535
 constexpr int kWarpsPerBlock = 2;
-constexpr uint32_t kSmemSlotLimit = 24u * 1024u;  // slots go to shared memory up to this many bytes per replica
+constexpr uint32_t kSmemSlotLimit = 25u * 1024u;  // slots go to shared memory up to this many bytes per replica
 constexpr uint32_t kMagicBytes = 528;             // ceil(2^64 / d) for d = 0..64, rounded up to 16 bytes
+constexpr uint32_t kHashSlots = 512;              // per-warp set of event times (C > 1 variants)
 
 enum : int { MIG_NONE = 0, MIG_SRC = 1, MIG_DST = 2 };
 
@@ -100,13 +101,14 @@ struct RepState {
 };
 
 struct Params {
-    int R, N, M, T, Bmax, BP, K, S, cap, enable_mig, theta_num, theta_den;
-    uint32_t NS;                  // slots per replica: N * BP rounded up to a multiple of 4 (whole 16-byte rows)
+    int R, N, M, T, Bmax, SP, K, S, cap, enable_mig, theta_num, theta_den;
+    uint32_t NS;                  // slots per replica: N * SP rounded up to a multiple of 4 (whole 16-byte rows)
     uint32_t interval, max_steps;
     unsigned long long magT;      // ceil(2^40 / T)
     int base, a, b;
     Layout L;
     uint32_t slot_bytes;          // NS * 12 when the slots live in shared memory, else 0
+    uint32_t hash_bytes;          // per-warp event-time set (C > 1 variants), else 0
     const long long *offsets;
     const uint32_t *arrival;
     const uint16_t *plen, *olen;
@@ -124,7 +126,10 @@ struct Params {
 
 // Per-warp view of the replica being simulated.  Pointers into shared memory
 // for instance state (and slots when they fit), into HBM for request state;
-// scalars are warp-uniform.
+// scalars are warp-uniform.  Instance i's slots are sst[i*SP + s], srid[i*SP + s]
+// with an odd stride SP, so one lane per instance walks its slots without
+// shared-memory bank conflicts; the cooperative paths give lane l slots l and
+// 32 + l.
 struct Ctx {
     uint32_t *busy, *mreq, *head, *tail;
     int *free_, *resv, *hol, *hr, *key, *mcopied, *h;
@@ -132,6 +137,7 @@ struct Ctx {
     uint8_t *nrun, *nb, *mrole, *mpeer;
     uint64_t *sst;
     uint32_t *srid;
+    uint32_t *tset;                   // event-time set (C > 1)
     const unsigned long long *magic;  // [65]: ceil(2^64 / d) for d >= 2
     const uint32_t *arrival;
     const uint16_t *plen, *olen;
@@ -141,13 +147,22 @@ struct Ctx {
     sim_request_result_t *res;
     sim_migration_event_t *log;
     unsigned long long magT;
-    int N, K, T, Bmax, BP, S, cap, lane;
+    int N, K, T, Bmax, SP, S, cap, lane;
     uint32_t Q, t;
 };
 
-// Counters.  `finished` is warp-uniform; the others are exact on lane 0.
+// Counters of the cooperative paths.  `finished` is warp-uniform; the others
+// are exact on lane 0.
 struct Cnt {
     uint32_t finished, log_events, migrations, preemptions, starts, aborts, steps, iterations;
+    uint64_t member_iterations, events;
+    int status;
+};
+
+// Per-lane counters of the lane-parallel path (summed over the warp when the
+// warp leaves the replica; `finished` after every window).
+struct Acc {
+    uint32_t finished, preemptions, iterations;
     uint64_t member_iterations, events;
     int status;
 };
@@ -210,7 +225,7 @@ __device__ __forceinline__ int arg_ext(const Ctx &x, uint32_t el, bool want_max,
     return __shfl_sync(kFull, bi, __ffs(eq) - 1);
 }
 
-// ---- lane-0 bookkeeping helpers (no collectives inside) --------------------
+// ---- single-thread bookkeeping helpers (no collectives inside) -------------
 __device__ __forceinline__ void cnt_inc(const Ctx &x, int i, int k) {
     if (x.cnt[i * x.K + k]++ == 0) x.hr[i] += x.h[k];
 }
@@ -233,20 +248,20 @@ __device__ __forceinline__ void push_front(const Ctx &x, int i, int k, uint32_t 
     x.head[b] = r;
     x.wmask[i] |= (uint16_t)(1u << k);
 }
-__device__ __forceinline__ uint32_t pop_front(const Ctx &x, int i, int k, Cnt &cn) {
+__device__ __forceinline__ uint32_t pop_front(const Ctx &x, int i, int k, int &status) {
     const int b = i * x.K + k;
     const uint32_t r = x.head[b];
-    if (r >= x.Q) { cn.status = SIM_ERR_INTERNAL; return kNone; }
+    if (r >= x.Q) { status = SIM_ERR_INTERNAL; return kNone; }
     const uint32_t nx = x.link[r].x;
     x.head[b] = nx;
     if (nx != kNone) x.link[nx].y = kNone;
     else { x.tail[b] = kNone; x.wmask[i] &= (uint16_t)~(1u << k); }
     return r;
 }
-__device__ __forceinline__ uint32_t pop_back(const Ctx &x, int i, int k, Cnt &cn) {
+__device__ __forceinline__ uint32_t pop_back(const Ctx &x, int i, int k, int &status) {
     const int b = i * x.K + k;
     const uint32_t r = x.tail[b];
-    if (r >= x.Q) { cn.status = SIM_ERR_INTERNAL; return kNone; }
+    if (r >= x.Q) { status = SIM_ERR_INTERNAL; return kNone; }
     const uint32_t pv = x.link[r].y;
     x.tail[b] = pv;
     if (pv != kNone) x.link[pv].x = kNone;
@@ -294,8 +309,63 @@ __device__ __forceinline__ void abort_mig(const Ctx &x, Cnt &cn, int s) {
     clear_mig(x, s, d);
 }
 
-// ---- collective steps -------------------------------------------------------
-// Lane l holds slots 2l and 2l+1 of an instance.
+// Recompute-style preemption bookkeeping of running request r (state word a)
+// on instance i: back to the front of its bucket keeping g; the caller frees
+// its blocks and handles a migration that r was part of.
+template <class A>
+__device__ __forceinline__ void preempt_common(const Ctx &x, A &acc, int i, uint32_t r, uint64_t a) {
+    const int tr = (int)s_tier(a);
+    x.g[r] = (uint16_t)(x.olen[r] - s_left(a));
+    const uint32_t old = x.wmask[i];
+    push_front(x, i, tr, r);
+    if ((old & ((1u << tr) - 1u)) == 0) x.hol[i] = blocks_for(x, s_ctx(a));  // now head of line
+    bump_pre(x, r);
+    acc.preemptions++;
+    acc.events++;
+}
+
+// Batch formation steps (ii) and (iii) for instance i holding n running
+// requests and fr free blocks: admission in (tier, FCFS) order while the head
+// of line fits, then the iteration starts (Sec. 2.2, Sec. 3.1).  Single thread.
+template <class A>
+__device__ __forceinline__ void admit_and_start(const Ctx &x, A &acc, int i, int n, int fr, int base, int a_us,
+                                                int b_us) {
+    const int n_decode = n;
+    int prefill = 0;
+    int nr = n;
+    while (nr < x.Bmax) {
+        const uint32_t wm = x.wmask[i];
+        if (!wm) break;
+        const int need = x.hol[i];
+        if (need > fr) break;
+        const int k = __ffs(wm) - 1;
+        const uint32_t r = pop_front(x, i, k, acc.status);
+        if (r == kNone) break;
+        const uint32_t P = x.plen[r], O = x.olen[r], gg = x.g[r];
+        x.sst[i * x.SP + nr] = s_make(P + gg, (uint32_t)need, O - gg, (uint32_t)k, gg == 0);
+        x.srid[i * x.SP + nr] = r;
+        ++nr;
+        fr -= need;
+        prefill += (int)(P + gg);
+        refresh_hol(x, i);
+    }
+    x.nrun[i] = (uint8_t)nr;
+    x.free_[i] = fr;
+    if (nr > 0) {
+        const long long end = (long long)x.t + base + (long long)a_us * prefill + (long long)b_us * n_decode;
+        if (end > 0xFFFFFFFELL) {
+            acc.status = SIM_ERR_OVERFLOW;
+        } else {
+            x.busy[i] = (uint32_t)end;
+            x.nb[i] = (uint8_t)nr;
+            acc.iterations++;
+            acc.member_iterations += (uint64_t)nr;
+        }
+    }
+}
+
+// ---- cooperative (whole-warp) steps -----------------------------------------
+// Lane l holds slots l and 32 + l of an instance.
 struct Slots {
     uint64_t a0, a1;
     uint32_t r0, r1;
@@ -304,34 +374,25 @@ struct Slots {
 
 __device__ __forceinline__ Slots load_slots(const Ctx &x, int i, int n) {
     Slots s;
-    const int i0 = 2 * x.lane;
-    s.v0 = i0 < n;
-    s.v1 = i0 + 1 < n;
-    s.a0 = s.a1 = 0ull;
-    s.r0 = s.r1 = kNone;
-    if (s.v0) {
-        const ulonglong2 v = *reinterpret_cast<const ulonglong2 *>(x.sst + i * x.BP + i0);
-        const uint2 w = *reinterpret_cast<const uint2 *>(x.srid + i * x.BP + i0);
-        s.a0 = v.x;
-        s.a1 = v.y;
-        s.r0 = w.x;
-        s.r1 = w.y;
-    }
+    const uint64_t *st = x.sst + i * x.SP;
+    const uint32_t *rd = x.srid + i * x.SP;
+    s.v0 = x.lane < n;
+    s.v1 = x.lane + 32 < n;
+    s.a0 = s.v0 ? st[x.lane] : 0ull;
+    s.r0 = s.v0 ? rd[x.lane] : kNone;
+    s.a1 = s.v1 ? st[x.lane + 32] : 0ull;
+    s.r1 = s.v1 ? rd[x.lane + 32] : kNone;
     return s;
-}
-
-__device__ __forceinline__ void store_states(const Ctx &x, int i, uint64_t a0, uint64_t a1) {
-    *reinterpret_cast<ulonglong2 *>(x.sst + i * x.BP + 2 * x.lane) = make_ulonglong2(a0, a1);
 }
 
 // Writes the slots whose keep flag is set at their compacted (stable) positions; returns the count.
 __device__ __forceinline__ int compact_slots(const Ctx &x, int i, const Slots &s, bool k0, bool k1) {
-    uint64_t *st = x.sst + i * x.BP;
-    uint32_t *rd = x.srid + i * x.BP;
+    uint64_t *st = x.sst + i * x.SP;
+    uint32_t *rd = x.srid + i * x.SP;
     const uint32_t q0 = __ballot_sync(kFull, k0), q1 = __ballot_sync(kFull, k1);
     const uint32_t below = (1u << x.lane) - 1u;
-    const int p0 = __popc(q0 & below) + __popc(q1 & below);
-    const int p1 = p0 + (k0 ? 1 : 0);
+    const int p0 = __popc(q0 & below);
+    const int p1 = __popc(q0) + __popc(q1 & below);
     __syncwarp();
     if (k0) { st[p0] = s.a0; rd[p0] = s.r0; }
     if (k1) { st[p1] = s.a1; rd[p1] = s.r1; }
@@ -342,17 +403,17 @@ __device__ __forceinline__ int compact_slots(const Ctx &x, int i, const Slots &s
 // Commit a fully copied running request from s to d (Sec. 3.5, Fig. 4).
 __device__ __forceinline__ void commit_mig(const Ctx &x, Cnt &cn, int s, int d, int pos, uint64_t a, uint32_t rid,
                                            const Slots &sl, int n) {
-    uint64_t *st = x.sst + s * x.BP;
-    uint32_t *rd = x.srid + s * x.BP;
-    const int i0 = 2 * x.lane, i1 = i0 + 1;
+    uint64_t *st = x.sst + s * x.SP;
+    uint32_t *rd = x.srid + s * x.SP;
+    const int i0 = x.lane, i1 = x.lane + 32;
     __syncwarp();
     if (sl.v0 && i0 > pos) { st[i0 - 1] = sl.a0; rd[i0 - 1] = sl.r0; }
     if (sl.v1 && i1 > pos) { st[i1 - 1] = sl.a1; rd[i1 - 1] = sl.r1; }
     __syncwarp();
     if (x.lane == 0) {
         const int nd = x.nrun[d];
-        x.sst[d * x.BP + nd] = a;
-        x.srid[d * x.BP + nd] = rid;
+        x.sst[d * x.SP + nd] = a;
+        x.srid[d * x.SP + nd] = rid;
         x.nrun[d] = (uint8_t)(nd + 1);
         x.nrun[s] = (uint8_t)(n - 1);
         const int blocks = (int)s_blocks(a);
@@ -383,10 +444,10 @@ __device__ __forceinline__ void migration_stage(const Ctx &x, Cnt &cn, int s) {
         __syncwarp();
         return;
     }
-    const int l = __ffs(h0 | h1) - 1;
-    const int j = ((h0 >> l) & 1u) ? 0 : 1;
+    const int j = h0 ? 0 : 1;
+    const int l = __ffs(h0 ? h0 : h1) - 1;
     const uint64_t a = __shfl_sync(kFull, j ? sl.a1 : sl.a0, l);
-    const int pos = 2 * l + j;
+    const int pos = 32 * j + l;
     const int blocks = (int)s_blocks(a);
     int commit = 0;
     if (x.lane == 0) {
@@ -410,8 +471,7 @@ __device__ __forceinline__ void migration_stage(const Ctx &x, Cnt &cn, int s) {
 __device__ __forceinline__ void complete_instance(const Ctx &x, Cnt &cn, int i) {
     const int n = x.nrun[i], nb = x.nb[i];
     Slots sl = load_slots(x, i, n);
-    const int i0 = 2 * x.lane;
-    const bool b0 = i0 < nb, b1 = i0 + 1 < nb;
+    const bool b0 = x.lane < nb, b1 = x.lane + 32 < nb;
     bool g0 = false, g1 = false;
     if (b0) {
         sl.a0 += kAdvance;
@@ -426,18 +486,19 @@ __device__ __forceinline__ void complete_instance(const Ctx &x, Cnt &cn, int i) 
     const bool f0 = b0 && s_left(sl.a0) == 0, f1 = b1 && s_left(sl.a1) == 0;
     const uint32_t firsts = __reduce_add_sync(kFull, (uint32_t)g0 + (uint32_t)g1);
     if (!__any_sync(kFull, f0 || f1)) {
-        if (b0) store_states(x, i, sl.a0, sl.a1);
+        uint64_t *st = x.sst + i * x.SP;
+        if (b0) st[x.lane] = sl.a0;
+        if (b1) st[x.lane + 32] = sl.a1;
     } else {
         const uint32_t m0 = __ballot_sync(kFull, f0), m1 = __ballot_sync(kFull, f1);
         if (f0) { x.res[sl.r0].finish_us = x.t; x.res[sl.r0].final_instance = (uint16_t)i; }
         if (f1) { x.res[sl.r1].finish_us = x.t; x.res[sl.r1].final_instance = (uint16_t)i; }
-        uint32_t lanes = m0 | m1;
-        while (lanes) {  // finished requests in batch order
-            const int l = __ffs(lanes) - 1;
-            lanes &= lanes - 1;
 #pragma unroll
-            for (int j = 0; j < 2; ++j) {
-                if (!(((j ? m1 : m0) >> l) & 1u)) continue;
+        for (int j = 0; j < 2; ++j) {  // finished requests in batch order
+            uint32_t lanes = j ? m1 : m0;
+            while (lanes) {
+                const int l = __ffs(lanes) - 1;
+                lanes &= lanes - 1;
                 const uint64_t a = __shfl_sync(kFull, j ? sl.a1 : sl.a0, l);
                 const uint32_t r = __shfl_sync(kFull, j ? sl.r1 : sl.r0, l);
                 if (x.lane == 0) {
@@ -574,7 +635,7 @@ __device__ __forceinline__ void migration_tick(const Ctx &x, Cnt &cn, int theta_
         if (has_wait) {
             if (x.lane == 0) {
                 const int k = 31 - __clz((unsigned)x.wmask[s]);
-                const uint32_t r = pop_back(x, s, k, cn);
+                const uint32_t r = pop_back(x, s, k, cn.status);
                 if (r != kNone) {
                     refresh_hol(x, s);
                     cnt_dec(x, s, k);
@@ -618,19 +679,6 @@ __device__ __forceinline__ void migration_tick(const Ctx &x, Cnt &cn, int theta_
     }
 }
 
-// Preemption of running request r (state word a) on instance i: recompute style.
-__device__ __forceinline__ void preempt_book(const Ctx &x, Cnt &cn, int i, uint32_t r, uint64_t a) {
-    const int tr = (int)s_tier(a);
-    x.g[r] = (uint16_t)(x.olen[r] - s_left(a));
-    const uint32_t old = x.wmask[i];
-    push_front(x, i, tr, r);
-    if ((old & ((1u << tr) - 1u)) == 0) x.hol[i] = blocks_for(x, s_ctx(a));  // now head of line
-    bump_pre(x, r);
-    cn.preemptions++;
-    cn.events++;
-    if (x.mrole[i] == MIG_SRC && x.mreq[i] == r) abort_mig(x, cn, i);
-}
-
 // Phase 4: batch formation at idle instance i (Sec. 2.2 continuous batching).
 __device__ __forceinline__ void form_batch(const Ctx &x, Cnt &cn, int i, int base, int a_us, int b_us) {
     int n = x.nrun[i];
@@ -643,14 +691,16 @@ __device__ __forceinline__ void form_batch(const Ctx &x, Cnt &cn, int i, int bas
         // (i) every running request gets the KV growth it needs
         if (total > 0) {
             fr -= total;
-            if (d0 | d1) store_states(x, i, sl.a0 + ((uint64_t)d0 << 16), sl.a1 + ((uint64_t)d1 << 16));
+            uint64_t *st = x.sst + i * x.SP;
+            if (d0) st[x.lane] = sl.a0 + ((uint64_t)d0 << 16);
+            if (d1) st[x.lane + 32] = sl.a1 + ((uint64_t)d1 << 16);
         }
     } else {
         // (i) grow in running order; when out of blocks, preempt the lowest
         // priority, newest running request (possibly the one growing).
         bool al0 = sl.v0, al1 = sl.v1;
         for (int idx = 0; idx < n; ++idx) {
-            const int l = idx >> 1, j = idx & 1;
+            const int l = idx & 31, j = idx >> 5;
             for (;;) {
                 if (!__shfl_sync(kFull, (int)(j ? al1 : al0), l)) break;
                 const uint64_t a = __shfl_sync(kFull, j ? sl.a1 : sl.a0, l);
@@ -670,55 +720,127 @@ __device__ __forceinline__ void form_batch(const Ctx &x, Cnt &cn, int i, int bas
                 const uint32_t rmax = __reduce_max_sync(kFull, max(c0, c1));
                 const uint32_t vm0 = __ballot_sync(kFull, al0 && t0 == tmax && sl.r0 == rmax);
                 const uint32_t vm1 = __ballot_sync(kFull, al1 && t1 == tmax && sl.r1 == rmax);
-                const int vl = vm0 ? __ffs(vm0) - 1 : __ffs(vm1) - 1;
                 const int vj = vm0 ? 0 : 1;
+                const int vl = __ffs(vm0 ? vm0 : vm1) - 1;
                 const uint64_t va = __shfl_sync(kFull, vj ? sl.a1 : sl.a0, vl);
                 fr += (int)s_blocks(va);
                 if (x.lane == vl) { if (vj) al1 = false; else al0 = false; }
-                if (x.lane == 0) preempt_book(x, cn, i, rmax, va);
+                if (x.lane == 0) {
+                    preempt_common(x, cn, i, rmax, va);
+                    if (x.mrole[i] == MIG_SRC && x.mreq[i] == rmax) abort_mig(x, cn, i);
+                }
                 __syncwarp();
                 if (vl == l && vj == j) break;
             }
         }
         n = compact_slots(x, i, sl, al0, al1);
     }
-    // (ii) admission in (tier, FCFS) order while the head of line fits; (iii) start the iteration.
-    if (x.lane == 0) {
-        const int n_decode = n;
-        int prefill = 0;
-        int nr = n;
-        while (nr < x.Bmax) {
-            const uint32_t wm = x.wmask[i];
-            if (!wm) break;
-            const int need = x.hol[i];
-            if (need > fr) break;
-            const int k = __ffs(wm) - 1;
-            const uint32_t r = pop_front(x, i, k, cn);
-            if (r == kNone) break;
-            const uint32_t P = x.plen[r], O = x.olen[r], gg = x.g[r];
-            x.sst[i * x.BP + nr] = s_make(P + gg, (uint32_t)need, O - gg, (uint32_t)k, gg == 0);
-            x.srid[i * x.BP + nr] = r;
-            ++nr;
-            fr -= need;
-            prefill += (int)(P + gg);
-            refresh_hol(x, i);
-        }
-        x.nrun[i] = (uint8_t)nr;
-        x.free_[i] = fr;
-        if (nr > 0) {
-            const long long end =
-                (long long)x.t + base + (long long)a_us * prefill + (long long)b_us * n_decode;
-            if (end > 0xFFFFFFFELL) {
-                cn.status = SIM_ERR_OVERFLOW;
-            } else {
-                x.busy[i] = (uint32_t)end;
-                x.nb[i] = (uint8_t)nr;
-                cn.iterations++;
-                cn.member_iterations += (uint64_t)nr;
+    if (x.lane == 0) admit_and_start(x, cn, i, n, fr, base, a_us, b_us);
+    __syncwarp();
+}
+
+// ---- lane-parallel path -------------------------------------------------------
+// One lane advances instance i, which is in no migration, through its
+// iteration end at t (phase 1) and the batch formation that follows at t
+// (phase 4).  Exactly the cooperative semantics; only this lane runs it.
+__device__ __forceinline__ void solo_event(const Ctx &x, Acc &acc, int i, int base, int a_us, int b_us) {
+    uint64_t *st = x.sst + i * x.SP;
+    uint32_t *rd = x.srid + i * x.SP;
+    const int n0 = x.nrun[i], nb = x.nb[i];
+    int fr = x.free_[i];
+    int w = 0, total = 0;
+    uint64_t grow = 0;  // bit w: the kept slot w needs more KV blocks
+    for (int s = 0; s < n0; ++s) {
+        uint64_t a = st[s];
+        if (s < nb) {
+            a += kAdvance;
+            if (a & kFirst) {
+                a ^= kFirst;
+                x.res[rd[s]].first_token_us = x.t;
+                acc.events++;
+            }
+            if (s_left(a) == 0) {  // finished: free its KV
+                const uint32_t r = rd[s];
+                x.res[r].finish_us = x.t;
+                x.res[r].final_instance = (uint16_t)i;
+                fr += (int)s_blocks(a);
+                cnt_dec(x, i, (int)s_tier(a));
+                acc.finished++;
+                acc.events++;
+                continue;
             }
         }
+        const int def = blocks_for(x, s_ctx(a)) - (int)s_blocks(a);
+        if (def > 0) {
+            grow |= 1ull << w;
+            total += def;
+        }
+        if (w != s) rd[w] = rd[s];
+        st[w++] = a;
     }
-    __syncwarp();
+    int n = w;
+    x.busy[i] = kNone;
+    if (total <= fr) {
+        fr -= total;
+        while (grow) {
+            const int s = __ffsll((long long)grow) - 1;
+            grow &= grow - 1;
+            const uint64_t a = st[s];
+            st[s] = a + ((uint64_t)(blocks_for(x, s_ctx(a)) - (int)s_blocks(a)) << 16);
+        }
+    } else {
+        // grow in running order, preempting the lowest-priority newest request when out of blocks
+        uint64_t alive = n >= 64 ? ~0ull : ((1ull << n) - 1ull);
+        for (int idx = 0; idx < n; ++idx) {
+            if (!((alive >> idx) & 1ull)) continue;
+            for (;;) {
+                const uint64_t a = st[idx];
+                const int def = blocks_for(x, s_ctx(a)) - (int)s_blocks(a);
+                if (def <= 0) break;
+                if (fr > 0) {
+                    const int gv = min(fr, def);
+                    fr -= gv;
+                    st[idx] = a + ((uint64_t)gv << 16);
+                    continue;
+                }
+                int v = -1;
+                uint32_t vt = 0, vr = 0;
+                for (uint64_t m = alive; m; m &= m - 1) {
+                    const int s = __ffsll((long long)m) - 1;
+                    const uint32_t ts = s_tier(st[s]), rs = rd[s];
+                    if (v < 0 || ts > vt || (ts == vt && rs > vr)) { v = s; vt = ts; vr = rs; }
+                }
+                const uint64_t va = st[v];
+                fr += (int)s_blocks(va);
+                alive &= ~(1ull << v);
+                preempt_common(x, acc, i, vr, va);
+                if (v == idx) break;
+            }
+        }
+        int k = 0;
+        for (int s = 0; s < n; ++s) {
+            if (!((alive >> s) & 1ull)) continue;
+            if (k != s) { st[k] = st[s]; rd[k] = rd[s]; }
+            ++k;
+        }
+        n = k;
+    }
+    admit_and_start(x, acc, i, n, fr, base, a_us, b_us);
+}
+
+// Number of distinct event times in a window: `u[j]` is the event time of this
+// lane's instance j (kNone if none); coupled-instance step times are added by
+// the caller.  C == 1 uses __match_any_sync; wider variants insert into a
+// per-warp open-addressing set of event times, cleared by the caller.
+__device__ __forceinline__ uint32_t tset_insert(const Ctx &x, uint32_t t) {
+    uint32_t h = (t * 0x9E3779B1u) >> 23;  // 9 bits: kHashSlots = 512
+    for (uint32_t probe = 0; probe < kHashSlots; ++probe) {
+        const uint32_t old = atomicCAS(&x.tset[h], kNone, t);
+        if (old == kNone) return 1u;
+        if (old == t) return 0u;
+        h = (h + 1u) & (kHashSlots - 1u);
+    }
+    return 0u;
 }
 
 __device__ __forceinline__ void copy16(unsigned char *dst, const unsigned char *src, uint32_t bytes, int lane) {
@@ -746,20 +868,74 @@ __device__ __forceinline__ void bind_blob(Ctx &x, const Layout &L, unsigned char
     x.h = reinterpret_cast<int *>(blob + L.h);
 }
 
+// Phase 1 restricted to the instances whose bit is set in `mask` (bit j =
+// instance lane*C + j): iteration ends at x.t, ascending index.  Collective.
+template <int C>
+__device__ __forceinline__ void complete_all(const Ctx &x, Cnt &cn, uint32_t mask, const Params &p) {
+    uint32_t hits = 0;
+#pragma unroll
+    for (int j = 0; j < C; ++j) {
+        const int i = x.lane * C + j;
+        if (((mask >> j) & 1u) && x.busy[i] == x.t) hits |= 1u << j;
+    }
+    uint32_t lanes = __ballot_sync(kFull, hits != 0);
+    while (lanes) {
+        const int l = __ffs(lanes) - 1;
+        lanes &= lanes - 1;
+        uint32_t h = C == 1 ? 1u : __shfl_sync(kFull, hits, l);
+        while (h) {
+            const int j = __ffs(h) - 1;
+            h &= h - 1;
+            complete_instance(x, cn, l * C + j);
+        }
+    }
+}
+
+// Phase 4 restricted to `mask`: batch formation at every idle instance with
+// work, ascending index.  Collective.
+template <int C>
+__device__ __forceinline__ void form_all(const Ctx &x, Cnt &cn, uint32_t mask, const Params &p) {
+    uint32_t want = 0;
+#pragma unroll
+    for (int j = 0; j < C; ++j) {
+        const int i = x.lane * C + j;
+        if (((mask >> j) & 1u) && x.busy[i] == kNone && (x.nrun[i] | x.wmask[i]) != 0) want |= 1u << j;
+    }
+    uint32_t lanes = __ballot_sync(kFull, want != 0);
+    while (lanes) {
+        const int l = __ffs(lanes) - 1;
+        lanes &= lanes - 1;
+        uint32_t h = C == 1 ? 1u : __shfl_sync(kFull, want, l);
+        while (h) {
+            const int j = __ffs(h) - 1;
+            h &= h - 1;
+            form_batch(x, cn, l * C + j, p.base, p.a, p.b);
+        }
+    }
+}
+
 // The persistent simulation kernel: each warp repeatedly takes a replica and
 // advances it by up to p.max_steps event times.  C = instances per lane;
 // SMS = running-request slots staged in shared memory.
+//
+// Between two global events (the next arrival, the next migration tick) the
+// instances that are in no migration do not interact, and an iteration lasts
+// at least `base` microseconds.  So in a window [tmin, min(T_g, tmin + base))
+// every instance ends at most one iteration, and the lanes advance their own
+// instances in parallel; instances in a migration, and every step at a global
+// event, go through the cooperative single-step code in time order.
 template <int C, bool SMS>
-__global__ void __launch_bounds__(32 * kWarpsPerBlock) k_run(Params p) {
+__global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
     extern __shared__ __align__(16) unsigned char smem[];
     unsigned long long *magic = reinterpret_cast<unsigned long long *>(smem);
     for (int d = threadIdx.x; d <= 64; d += blockDim.x)
         magic[d] = d < 2 ? 0ull : ~0ull / (unsigned long long)d + 1ull;
     __syncthreads();
     const int lane = threadIdx.x & 31;
-    const uint32_t per_warp = p.L.bytes + p.slot_bytes;
+    const uint32_t per_warp = p.L.bytes + p.slot_bytes + p.hash_bytes;
     unsigned char *blob = smem + kMagicBytes + (size_t)(threadIdx.x >> 5) * per_warp;
     unsigned char *sslots = blob + p.L.bytes;
+    uint32_t *tset = reinterpret_cast<uint32_t *>(blob + p.L.bytes + p.slot_bytes);
     const uint32_t nslot = p.NS;
     for (;;) {
         int r = 0;
@@ -783,6 +959,7 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock) k_run(Params p) {
             x.sst = g_sst;
             x.srid = g_srid;
         }
+        x.tset = tset;
         __syncwarp();
         const long long o = p.offsets[r];
         x.Q = (uint32_t)(p.offsets[r + 1] - o);
@@ -800,7 +977,7 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock) k_run(Params p) {
         x.K = p.K;
         x.T = p.T;
         x.Bmax = p.Bmax;
-        x.BP = p.BP;
+        x.SP = p.SP;
         x.S = p.S;
         x.cap = p.cap;
         x.lane = lane;
@@ -817,16 +994,23 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock) k_run(Params p) {
         cn.member_iterations = rs.member_iterations;
         cn.events = rs.events;
         cn.status = SIM_REPLICA_RUNNING;
+        Acc acc;
+        acc.finished = 0;
+        acc.preemptions = 0;
+        acc.iterations = 0;
+        acc.member_iterations = 0;
+        acc.events = 0;
+        acc.status = 0;
         uint32_t cursor = rs.cursor;
         uint32_t next_tick = rs.next_tick;
         ArrBuf ab;
         arr_refill(x, ab, cursor);
         uint32_t next_arr = __shfl_sync(kFull, ab.time, 0);
         const uint32_t max_steps = p.max_steps;
+        const uint32_t all = own_mask<C>(x);
         for (;;) {
             if (cn.finished == x.Q) { cn.status = SIM_REPLICA_DONE; break; }
             if (cn.steps == max_steps) break;
-            // a0: next event time
             uint32_t bz[C];
             uint32_t mb = kNone;
 #pragma unroll
@@ -836,61 +1020,112 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock) k_run(Params p) {
                 mb = min(mb, bz[j]);
             }
             const uint32_t tb = __reduce_min_sync(kFull, mb);
+            const uint32_t tg = p.enable_mig ? min(next_arr, next_tick) : next_arr;
+            if (tb < tg && max_steps - cn.steps > (uint32_t)x.N) {
+                // ---- window [tb, t1): at most one iteration end per instance ----
+                const uint32_t t1 = (uint32_t)min((unsigned long long)tg, (unsigned long long)tb + (uint32_t)p.base);
+                uint32_t cm = 0, solo = 0;  // instances with an iteration end in the window: in a migration / not
+#pragma unroll
+                for (int j = 0; j < C; ++j) {
+                    const int i = lane * C + j;
+                    if (bz[j] < t1) {
+                        if (x.mrole[i] != MIG_NONE) cm |= 1u << j; else solo |= 1u << j;
+                    }
+                }
+                if (C > 1) {
+                    for (uint32_t q = (uint32_t)lane; q < kHashSlots; q += 32) tset[q] = kNone;
+                    __syncwarp();
+                }
+                uint32_t fresh = 0;   // distinct event times this lane contributes
+                uint32_t tlast = 0;   // latest event time processed in the window
+                if (solo) {
+#pragma unroll
+                    for (int j = 0; j < C; ++j) {
+                        if (!((solo >> j) & 1u)) continue;
+                        x.t = bz[j];
+                        tlast = max(tlast, bz[j]);
+                        if (C > 1) fresh += tset_insert(x, bz[j]);
+                        solo_event(x, acc, lane * C + j, p.base, p.a, p.b);
+                    }
+                }
+                __syncwarp();
+                uint32_t ucount;
+                uint32_t u = kNone;
+                if (C == 1) {
+                    u = solo ? bz[0] : kNone;
+                    const uint32_t grp = __match_any_sync(kFull, u);
+                    ucount = __popc(__ballot_sync(kFull, u != kNone && (__ffs(grp) - 1) == lane));
+                } else {
+                    ucount = __reduce_add_sync(kFull, fresh);
+                }
+                // instances in a migration (both ends, with or without an event of
+                // their own in the window): cooperative steps in time order
+                if (__any_sync(kFull, cm != 0)) {
+#pragma unroll
+                    for (int j = 0; j < C; ++j) {
+                        const int i = lane * C + j;
+                        if (i < x.N && x.mrole[i] != MIG_NONE) cm |= 1u << j;
+                    }
+                    for (;;) {
+                        uint32_t cb = kNone;
+#pragma unroll
+                        for (int j = 0; j < C; ++j) {
+                            const int i = lane * C + j;
+                            if ((cm >> j) & 1u) cb = min(cb, x.busy[i]);
+                        }
+                        const uint32_t tc = __reduce_min_sync(kFull, cb);
+                        if (tc >= t1) break;
+                        x.t = tc;
+                        tlast = max(tlast, tc);
+                        complete_all<C>(x, cn, cm, p);
+                        form_all<C>(x, cn, cm, p);
+                        if (C == 1) {
+                            ucount += __any_sync(kFull, u == tc) ? 0u : 1u;
+                        } else {
+                            uint32_t f2 = 0;
+                            if (lane == 0) f2 = tset_insert(x, tc);
+                            ucount += __shfl_sync(kFull, f2, 0);
+                        }
+                        cn.status = __shfl_sync(kFull, cn.status, 0);
+                        if (cn.status < 0) break;
+                    }
+                }
+                cn.steps += ucount;
+                x.t = __reduce_max_sync(kFull, tlast);
+                cn.finished += __reduce_add_sync(kFull, acc.finished);
+                acc.finished = 0;
+                const int ws = __reduce_min_sync(kFull, acc.status);
+                if (ws < 0 && cn.status >= 0) cn.status = ws;
+                if (cn.status < 0) break;
+                continue;
+            }
+            // ---- one step at the next event time (global events, or near the step limit) ----
             const uint32_t tc = min(tb, next_arr);
             if (tc == kNone) { cn.status = SIM_ERR_DEADLOCK; break; }
             const bool tick = p.enable_mig && next_tick <= tc;
             x.t = tick ? next_tick : tc;
             ++cn.steps;
-            // 1. iteration ends, ascending instance index
-            if (tb == x.t) {
-                uint32_t hits = 0;
-#pragma unroll
-                for (int j = 0; j < C; ++j)
-                    if (bz[j] == x.t) hits |= 1u << j;
-                uint32_t lanes = __ballot_sync(kFull, hits != 0);
-                while (lanes) {
-                    const int l = __ffs(lanes) - 1;
-                    lanes &= lanes - 1;
-                    uint32_t h = C == 1 ? 1u : __shfl_sync(kFull, hits, l);
-                    while (h) {
-                        const int j = __ffs(h) - 1;
-                        h &= h - 1;
-                        complete_instance(x, cn, l * C + j);
-                    }
-                }
-            }
-            // 2. dispatch of arrivals at t
-            if (next_arr == x.t) dispatch_phase<C>(x, cn, cursor, next_arr, ab);
-            // 3. migration tick
-            if (tick) {
+            if (tb == x.t) complete_all<C>(x, cn, all, p);  // 1. iteration ends
+            if (next_arr == x.t) dispatch_phase<C>(x, cn, cursor, next_arr, ab);  // 2. dispatch
+            if (tick) {  // 3. migration tick
                 const uint32_t nt = next_tick + p.interval;
                 next_tick = nt < next_tick ? kNone : nt;  // saturate: no tick beyond 2^32 - 1
                 migration_tick<C>(x, cn, p.theta_num, p.theta_den);
             }
-            // 4. batch formation at idle instances with work, ascending index
-            {
-                uint32_t want = 0;
-#pragma unroll
-                for (int j = 0; j < C; ++j) {
-                    const int i = lane * C + j;
-                    if (i < x.N && x.busy[i] == kNone && (x.nrun[i] | x.wmask[i]) != 0) want |= 1u << j;
-                }
-                uint32_t lanes = __ballot_sync(kFull, want != 0);
-                while (lanes) {
-                    const int l = __ffs(lanes) - 1;
-                    lanes &= lanes - 1;
-                    uint32_t h = C == 1 ? 1u : __shfl_sync(kFull, want, l);
-                    while (h) {
-                        const int j = __ffs(h) - 1;
-                        h &= h - 1;
-                        form_batch(x, cn, l * C + j, p.base, p.a, p.b);
-                    }
-                }
-            }
+            form_all<C>(x, cn, all, p);  // 4. batch formation
             cn.status = __shfl_sync(kFull, cn.status, 0);
             if (cn.status < 0) break;
         }
         __syncwarp();
+        // fold the lane-parallel counters into lane 0's
+        const uint32_t a_pre = __reduce_add_sync(kFull, acc.preemptions);
+        const uint32_t a_it = __reduce_add_sync(kFull, acc.iterations);
+        uint64_t a_mi = acc.member_iterations, a_ev = acc.events;
+#pragma unroll
+        for (int sh = 16; sh > 0; sh >>= 1) {
+            a_mi += __shfl_xor_sync(kFull, a_mi, sh);
+            a_ev += __shfl_xor_sync(kFull, a_ev, sh);
+        }
         copy16(gblob, blob, p.L.bytes, lane);
         if (SMS) {
             copy16(reinterpret_cast<unsigned char *>(g_sst), sslots, nslot * 8, lane);
@@ -905,11 +1140,11 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock) k_run(Params p) {
             o2.next_tick = next_tick;
             o2.pad0 = 0;
             o2.steps = rs.steps + cn.steps;
-            o2.iterations = rs.iterations + cn.iterations;
-            o2.member_iterations = cn.member_iterations;
-            o2.events = cn.events;
+            o2.iterations = rs.iterations + cn.iterations + a_it;
+            o2.member_iterations = cn.member_iterations + a_mi;
+            o2.events = cn.events + a_ev;
             o2.migrations = cn.migrations;
-            o2.preemptions = cn.preemptions;
+            o2.preemptions = cn.preemptions + a_pre;
             o2.starts = cn.starts;
             o2.aborts = cn.aborts;
             o2.status = cn.status;
@@ -1016,7 +1251,7 @@ __global__ void k_export_stats(const RepState *rep, sim_replica_stats_t *out, in
 typedef void (*RunKernel)(Params);
 
 template <bool SMS>
-RunKernel pick(int c) {
+RunKernel pick(int c) {  // c = instances per lane
     switch (c) {
         case 1: return k_run<1, SMS>;
         case 2: return k_run<2, SMS>;
@@ -1065,15 +1300,18 @@ inline Layout make_layout(int N, int K) {
 }
 
 // Chooses the kernel variant and grid for a problem; cudaSuccess or the error.
-inline uint32_t slots_per_replica(int N, int BP) { return ((uint32_t)N * (uint32_t)BP + 3u) & ~3u; }
+// Odd slot stride per instance (>= Bmax), so lanes walking different instances hit different banks.
+inline int slot_stride(int Bmax) { return Bmax | 1; }
+inline uint32_t slots_per_replica(int N, int SP) { return ((uint32_t)N * (uint32_t)SP + 3u) & ~3u; }
+inline uint32_t hash_bytes_for(int N) { return lanes_c(N) > 1 ? kHashSlots * 4u : 0u; }
 
-inline cudaError_t plan_launch(int R, int N, int BP, const Layout &L, Launch &out) {
+inline cudaError_t plan_launch(int R, int N, int SP, const Layout &L, Launch &out) {
     const int c = lanes_c(N);
-    const uint32_t slots = slots_per_replica(N, BP) * 12u;
+    const uint32_t slots = slots_per_replica(N, SP) * 12u;
     const bool sms = slots <= kSmemSlotLimit;
     out.fn = sms ? pick<true>(c) : pick<false>(c);
     out.slot_bytes = sms ? slots : 0u;
-    out.smem = kMagicBytes + (size_t)kWarpsPerBlock * (L.bytes + out.slot_bytes);
+    out.smem = kMagicBytes + (size_t)kWarpsPerBlock * (L.bytes + out.slot_bytes + hash_bytes_for(N));
     int dev = 0, sms_count = 0, per_sm = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms_count, cudaDevAttrMultiProcessorCount, dev);
@@ -1098,7 +1336,7 @@ inline unsigned long long magic40(unsigned d) { return ((1ull << kMagicShift) + 
 struct sim {
     sim_cluster_t cl;
     sim_policy_t pol;
-    int K = 0, ntables = 0, BP = 0;
+    int K = 0, ntables = 0, SP = 0;
     std::vector<int> tbl_k, tbl_h, rep_table;
     cudaStream_t stream = nullptr;
     sim_allocator_t al{};
@@ -1184,8 +1422,8 @@ void fill_scalars(mt::Params &p, const sim_cluster_t &cl, const sim_policy_t &po
     p.M = cl.blocks_per_instance;
     p.T = cl.tokens_per_block;
     p.Bmax = cl.max_batch;
-    p.BP = (cl.max_batch + 1) & ~1;
-    p.NS = mt::slots_per_replica(cl.num_instances, p.BP);
+    p.SP = mt::slot_stride(cl.max_batch);
+    p.NS = mt::slots_per_replica(cl.num_instances, p.SP);
     p.K = K;
     p.S = pol.migrate_blocks_per_iter;
     p.cap = cap;
@@ -1200,6 +1438,7 @@ void fill_scalars(mt::Params &p, const sim_cluster_t &cl, const sim_policy_t &po
     p.b = (int)pol.iter_us_per_decode_seq;
     p.L = L;
     p.slot_bytes = slot_bytes;
+    p.hash_bytes = mt::hash_bytes_for(cl.num_instances);
 }
 
 mt::Params make_params(const sim_t *s, long long max_steps) {
@@ -1278,9 +1517,9 @@ int validate_config(sim_t *s, const sim_cluster_t *cl, const sim_tier_table_t *t
     if (pol->enable_migration != 0 && pol->enable_migration != 1)
         return fail(s, SIM_ERR_ARG, "enable_migration must be 0 or 1");
     const long long lim24 = 1LL << 24;
-    if (pol->iter_base_us < 0 || pol->iter_base_us > lim24 || pol->iter_us_per_prefill_token < 0 ||
+    if (pol->iter_base_us < 1 || pol->iter_base_us > lim24 || pol->iter_us_per_prefill_token < 0 ||
         pol->iter_us_per_prefill_token > lim24 || pol->iter_us_per_decode_seq < 0 || pol->iter_us_per_decode_seq > lim24)
-        return fail(s, SIM_ERR_ARG, "iteration-time coefficients must be in [0, 2^24]");
+        return fail(s, SIM_ERR_ARG, "iteration-time base must be in [1, 2^24], the other coefficients in [0, 2^24]");
     if (pol->migrate_blocks_per_iter < 1 || pol->migrate_blocks_per_iter > 65535)
         return fail(s, SIM_ERR_ARG, "migrate_blocks_per_iter must be in [1, 65535]");
     if (pol->theta_den < 1 || pol->theta_num < 0 || pol->theta_num > (1 << 20) || pol->theta_den > (1 << 20))
@@ -1330,7 +1569,7 @@ int sim_create(const sim_cluster_t *cl, const sim_tier_table_t *tt, const sim_po
     s->pol = *pol;
     s->K = tt->max_tiers;
     s->ntables = tt->num_tables;
-    s->BP = (cl->max_batch + 1) & ~1;
+    s->SP = mt::slot_stride(cl->max_batch);
     s->tbl_k.assign(tt->num_tiers, tt->num_tiers + tt->num_tables);
     s->tbl_h.assign(tt->headroom_blocks, tt->headroom_blocks + (size_t)tt->num_tables * tt->max_tiers);
     s->rep_table.assign(tt->replica_table, tt->replica_table + cl->num_replicas);
@@ -1338,7 +1577,7 @@ int sim_create(const sim_cluster_t *cl, const sim_tier_table_t *tt, const sim_po
     if (allocator) { s->al = *allocator; s->use_al = true; }
     s->L = mt::make_layout(cl->num_instances, s->K);
 
-    const size_t R = (size_t)cl->num_replicas, NS = mt::slots_per_replica(cl->num_instances, s->BP);
+    const size_t R = (size_t)cl->num_replicas, NS = mt::slots_per_replica(cl->num_instances, s->SP);
     s->d_rep_table = (int *)dalloc(s, R * 4);
     s->d_tbl_k = (int *)dalloc(s, (size_t)s->ntables * 4);
     s->d_tbl_h = (int *)dalloc(s, (size_t)s->ntables * s->K * 4);
@@ -1363,7 +1602,7 @@ int sim_create(const sim_cluster_t *cl, const sim_tier_table_t *tt, const sim_po
     int dev = 0;
     if (e == cudaSuccess) e = cudaGetDevice(&dev);
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&s->sms, cudaDevAttrMultiProcessorCount, dev);
-    if (e == cudaSuccess) e = mt::plan_launch(cl->num_replicas, cl->num_instances, s->BP, s->L, s->launch);
+    if (e == cudaSuccess) e = mt::plan_launch(cl->num_replicas, cl->num_instances, s->SP, s->L, s->launch);
     if (e != cudaSuccess) {
         cudaGetLastError();
         rc = e == cudaErrorInvalidConfiguration
@@ -1563,11 +1802,11 @@ extern "C" int sim_run_static(const sim_cluster_t *cl, const sim_tier_table_t *t
     const int cap = events ? pol->event_log_capacity : 0;
 
     // Carve the scratch array.
-    const int N = cl->num_instances, BP = (cl->max_batch + 1) & ~1, K = tt->max_tiers;
+    const int N = cl->num_instances, SP = mt::slot_stride(cl->max_batch), K = tt->max_tiers;
     const mt::Layout L = mt::make_layout(N, K);
     size_t o = 0;
     const size_t o_blobs = o; o = align256(o + (size_t)R * L.bytes);
-    const size_t NS = mt::slots_per_replica(N, BP);
+    const size_t NS = mt::slots_per_replica(N, SP);
     const size_t o_srid = o; o = align256(o + (size_t)R * NS * 4);
     const size_t o_sst = o; o = align256(o + (size_t)R * NS * 8);
     const size_t o_rep = o; o = align256(o + (size_t)R * sizeof(mt::RepState));
@@ -1597,7 +1836,7 @@ extern "C" int sim_run_static(const sim_cluster_t *cl, const sim_tier_table_t *t
     cudaStream_t st = (cudaStream_t)cuda_stream;
 
     mt::Launch lc;
-    e = mt::plan_launch(R, N, BP, L, lc);
+    e = mt::plan_launch(R, N, SP, L, lc);
     if (e != cudaSuccess) {
         cudaGetLastError();
         return e == cudaErrorInvalidConfiguration
