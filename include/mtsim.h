@@ -89,7 +89,7 @@ typedef struct {
     int32_t num_replicas;        /* R >= 1 */
     int32_t num_instances;       /* N in [1, SIM_MAX_INSTANCES] */
     int32_t blocks_per_instance; /* M in [1, SIM_MAX_BLOCKS] KV blocks per instance */
-    int32_t tokens_per_block;    /* T in [1, 65535] */
+    int32_t tokens_per_block;    /* T in [1, 64] tokens per KV block */
     int32_t max_batch;           /* Bmax in [1, SIM_MAX_BATCH] running requests per instance */
 } sim_cluster_t;
 
@@ -106,9 +106,9 @@ typedef struct {
 typedef struct {
     int32_t policy;                     /* SIM_POLICY_LLUMNIX_MT */
     int32_t enable_migration;           /* 0 or 1 */
-    int64_t iter_base_us;               /* iteration time = base */
+    int64_t iter_base_us;               /* iteration time = base, in [1, 2^24] */
     int64_t iter_us_per_prefill_token;  /*   + a * prefill tokens in the batch */
-    int64_t iter_us_per_decode_seq;     /*   + b * decode requests in the batch; each in [0, 2^24] */
+    int64_t iter_us_per_decode_seq;     /*   + b * decode requests in the batch; a, b in [0, 2^24] */
     int32_t migrate_blocks_per_iter;    /* S: KV blocks copied per source iteration, in [1, 65535] */
     int32_t theta_num, theta_den;       /* imbalance threshold theta = num/den (0.3 = 3/10) */
     int32_t event_log_capacity;         /* migration-log records kept per replica, in [0, 2^24] */

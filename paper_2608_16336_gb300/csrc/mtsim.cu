@@ -62,31 +62,37 @@ constexpr int kKeyShift = 12;            // keys are floor(num * 4096 / den)
 constexpr int kMaxKeyRange = 1 << 19;    // |num| < 2^19 keeps num * 4096 below 2^31
 constexpr int kMagicShift = 40;          // floor(n / T) = (n * ceil(2^40 / T)) >> 40 for n < 2^20, T <= 65535
 constexpr int kWarpsPerBlock = 2;
-constexpr uint32_t kSmemSlotLimit = 25u * 1024u;  // slots go to shared memory up to this many bytes per replica
-constexpr uint32_t kMagicBytes = 528;             // ceil(2^64 / d) for d = 0..64, rounded up to 16 bytes
-constexpr uint32_t kHashSlots = 512;              // per-warp set of event times (C > 1 variants)
+constexpr int kMaxBlockTokens = 64;      // T limit of the per-instance growth histogram
+constexpr uint32_t kMagicBytes = 528;    // ceil(2^64 / d) for d = 0..64, rounded up to 16 bytes
+constexpr uint32_t kHashSlots = 512;     // per-warp set of event times (C > 1 variants)
 
 enum : int { MIG_NONE = 0, MIG_SRC = 1, MIG_DST = 2 };
 
-// Slot state word: ctx (P + g) | blocks << 16 | left (O - g) << 32 | tier << 48 | flags << 56.
-constexpr uint64_t kFirst = 1ull << 56;             // first token not produced yet
-constexpr uint64_t kAdvance = 1ull - (1ull << 32);  // ctx + 1, left - 1
-__device__ __forceinline__ uint32_t s_ctx(uint64_t s) { return (uint32_t)s & 0xFFFFu; }
-__device__ __forceinline__ uint32_t s_blocks(uint64_t s) { return (uint32_t)s >> 16; }
-__device__ __forceinline__ uint32_t s_left(uint64_t s) { return (uint32_t)(s >> 32) & 0xFFFFu; }
-__device__ __forceinline__ uint32_t s_tier(uint64_t s) { return (uint32_t)(s >> 48) & 0xFFu; }
-__device__ __forceinline__ uint64_t s_make(uint32_t ctx, uint32_t blocks, uint32_t left, uint32_t tier, bool first) {
-    return (uint64_t)(ctx | (blocks << 16)) | ((uint64_t)(left | (tier << 16)) << 32) | (first ? kFirst : 0ull);
-}
+// A running request is a 16-byte slot record, written when it joins an
+// instance's running list and read only on events (finish, preemption,
+// migration, first token):
+//   x = request id (index in the replica's trace)
+//   y = phi: number of the instance's first formation that includes it
+//   z = c | left << 16: its context length P + g and its remaining output O - g at formation phi
+//   w = tier | flags << 8 | rho << 16, rho = (c - phi) mod T
+// With nf formations done and pc = 1 after the iteration that followed the
+// last one (0 before), the request has advanced adv = nf - phi + pc tokens
+// (0 if phi > nf) and holds ceil((c + nf - phi) / T) KV blocks: every
+// formation grows each surviving request to exactly its need, one block at a
+// time because contexts grow by one token per iteration.  So the number of
+// requests that need a new block at the next formation is the count of
+// running requests with rho == -nf (mod T), and a request finishes at the
+// iteration that follows formation phi + left - 1.
+constexpr uint32_t kFirstFlag = 1u << 8;  // fresh request: its first token is due at the next iteration end
 
-// Byte offsets of the per-replica state blob (identical in HBM and shared memory).
 struct Layout {
-    uint32_t busy, free_, resv, hol, hr, key, mreq, mcopied;  // [N] x 4 B
-    uint32_t wmask;                                           // [N] x 2 B
-    uint32_t nrun, nb, mrole, mpeer;                          // [N] x 1 B
-    uint32_t cnt;                                             // [N*K] x 2 B
-    uint32_t head, tail;                                      // [N*K] x 4 B
-    uint32_t h;                                               // [K] x 4 B
+    uint32_t busy, free_, resv, hol, hr, key, mreq, mcopied, nf, minfin;  // [N] x 4 B
+    uint32_t wmask;                                                      // [N] x 2 B
+    uint32_t nrun, pc, phase, alo, ahi, mrole, mpeer;                     // [N] x 1 B
+    uint32_t cnt;                                                        // [N*K] x 2 B
+    uint32_t head, tail;                                                 // [N*K] x 4 B
+    uint32_t h;                                                          // [K] x 4 B
+    uint32_t hist;                                                       // [N*TH] x 1 B
     uint32_t bytes;
 };
 
@@ -101,13 +107,11 @@ struct RepState {
 };
 
 struct Params {
-    int R, N, M, T, Bmax, SP, K, S, cap, enable_mig, theta_num, theta_den;
-    uint32_t NS;                  // slots per replica: N * SP rounded up to a multiple of 4 (whole 16-byte rows)
+    int R, N, M, T, TH, Bmax, K, S, cap, enable_mig, theta_num, theta_den;
     uint32_t interval, max_steps;
     unsigned long long magT;      // ceil(2^40 / T)
     int base, a, b;
     Layout L;
-    uint32_t slot_bytes;          // NS * 12 when the slots live in shared memory, else 0
     uint32_t hash_bytes;          // per-warp event-time set (C > 1 variants), else 0
     const long long *offsets;
     const uint32_t *arrival;
@@ -117,26 +121,21 @@ struct Params {
     uint2 *link;  // .x = next, .y = prev
     sim_request_result_t *res;
     unsigned char *blobs;
-    uint32_t *srid;
-    uint64_t *sst;
+    uint4 *slots;                 // [R][N][Bmax]
     RepState *rep;
     sim_migration_event_t *log;
     int *work;
 };
 
-// Per-warp view of the replica being simulated.  Pointers into shared memory
-// for instance state (and slots when they fit), into HBM for request state;
-// scalars are warp-uniform.  Instance i's slots are sst[i*SP + s], srid[i*SP + s]
-// with an odd stride SP, so one lane per instance walks its slots without
-// shared-memory bank conflicts; the cooperative paths give lane l slots l and
-// 32 + l.
+// Per-warp view of the replica being simulated: instance state in shared
+// memory, request state and slot records in HBM; scalars are warp-uniform
+// except t while lanes advance their own instances.
 struct Ctx {
-    uint32_t *busy, *mreq, *head, *tail;
+    uint32_t *busy, *mreq, *head, *tail, *nf, *minfin;
     int *free_, *resv, *hol, *hr, *key, *mcopied, *h;
     uint16_t *wmask, *cnt;
-    uint8_t *nrun, *nb, *mrole, *mpeer;
-    uint64_t *sst;
-    uint32_t *srid;
+    uint8_t *nrun, *pc, *phase, *alo, *ahi, *mrole, *mpeer, *hist;
+    uint4 *slots;
     uint32_t *tset;                   // event-time set (C > 1)
     const unsigned long long *magic;  // [65]: ceil(2^64 / d) for d >= 2
     const uint32_t *arrival;
@@ -147,28 +146,27 @@ struct Ctx {
     sim_request_result_t *res;
     sim_migration_event_t *log;
     unsigned long long magT;
-    int N, K, T, Bmax, SP, S, cap, lane;
+    int N, K, T, TH, Bmax, S, cap, lane;
     uint32_t Q, t;
 };
 
-// Counters of the cooperative paths.  `finished` is warp-uniform; the others
-// are exact on lane 0.
+// Counters.  Lane 0's copy carries the replica's totals; the other lanes'
+// copies collect what they add while advancing their own instances and are
+// folded into lane 0's when the warp leaves the replica (`finished` after
+// every window).
 struct Cnt {
     uint32_t finished, log_events, migrations, preemptions, starts, aborts, steps, iterations;
     uint64_t member_iterations, events;
     int status;
 };
 
-// Per-lane counters of the lane-parallel path (summed over the warp when the
-// warp leaves the replica; `finished` after every window).
-struct Acc {
-    uint32_t finished, preemptions, iterations;
-    uint64_t member_iterations, events;
-    int status;
-};
-
 __device__ __forceinline__ int blocks_for(const Ctx &x, uint32_t tokens) {
     return (int)(((unsigned long long)(tokens + (uint32_t)x.T - 1u) * x.magT) >> kMagicShift);
+}
+__device__ __forceinline__ uint32_t mod_t(const Ctx &x, uint32_t v) {  // v mod T for v < 2^20
+    const uint32_t q = (uint32_t)(((unsigned long long)v * x.magT) >> kMagicShift);
+    const uint32_t r = v - q * (uint32_t)x.T;
+    return r >= (uint32_t)x.T ? r - (uint32_t)x.T : r;
 }
 
 // floor(v / d) for v < 2^32 and 1 <= d <= 64: the high half of v * ceil(2^64 / d).
@@ -225,7 +223,7 @@ __device__ __forceinline__ int arg_ext(const Ctx &x, uint32_t el, bool want_max,
     return __shfl_sync(kFull, bi, __ffs(eq) - 1);
 }
 
-// ---- single-thread bookkeeping helpers (no collectives inside) -------------
+// ---- single-thread instance logic (no collectives inside) -------------------
 __device__ __forceinline__ void cnt_inc(const Ctx &x, int i, int k) {
     if (x.cnt[i * x.K + k]++ == 0) x.hr[i] += x.h[k];
 }
@@ -309,219 +307,248 @@ __device__ __forceinline__ void abort_mig(const Ctx &x, Cnt &cn, int s) {
     clear_mig(x, s, d);
 }
 
-// Recompute-style preemption bookkeeping of running request r (state word a)
-// on instance i: back to the front of its bucket keeping g; the caller frees
-// its blocks and handles a migration that r was part of.
-template <class A>
-__device__ __forceinline__ void preempt_common(const Ctx &x, A &acc, int i, uint32_t r, uint64_t a) {
-    const int tr = (int)s_tier(a);
-    x.g[r] = (uint16_t)(x.olen[r] - s_left(a));
-    const uint32_t old = x.wmask[i];
-    push_front(x, i, tr, r);
-    if ((old & ((1u << tr) - 1u)) == 0) x.hol[i] = blocks_for(x, s_ctx(a));  // now head of line
-    bump_pre(x, r);
-    acc.preemptions++;
-    acc.events++;
+// Derived quantities of a slot record on instance i.
+__device__ __forceinline__ uint32_t sl_c(const uint4 &sl) { return sl.z & 0xFFFFu; }
+__device__ __forceinline__ uint32_t sl_left(const uint4 &sl) { return sl.z >> 16; }
+__device__ __forceinline__ uint32_t sl_tier(const uint4 &sl) { return sl.w & 0xFFu; }
+__device__ __forceinline__ uint32_t sl_rho(const uint4 &sl) { return sl.w >> 16; }
+__device__ __forceinline__ uint32_t sl_fin(const uint4 &sl) { return sl.y + sl_left(sl) - 1u; }
+__device__ __forceinline__ uint32_t sl_adv(const Ctx &x, int i, const uint4 &sl) {
+    const uint32_t nf = x.nf[i];
+    return sl.y <= nf ? nf - sl.y + x.pc[i] : 0u;
+}
+__device__ __forceinline__ int sl_blocks(const Ctx &x, int i, const uint4 &sl) {
+    return blocks_for(x, sl_c(sl) + x.nf[i] - sl.y);
+}
+__device__ __forceinline__ uint4 *slot_ptr(const Ctx &x, int i, int s) { return x.slots + i * x.Bmax + s; }
+
+// A request joins instance i's running list at position n with context c and
+// remaining output left; its first formation there will be number nf + 1.
+__device__ __forceinline__ void slot_join(const Ctx &x, int i, int n, uint32_t r, uint32_t c, uint32_t left,
+                                          uint32_t tier, bool fresh) {
+    const uint32_t phi = x.nf[i] + 1u;
+    const uint32_t pm = x.phase[i] + 1u == (uint32_t)x.T ? 0u : x.phase[i] + 1u;  // phi mod T
+    const uint32_t cm = mod_t(x, c);
+    const uint32_t rho = cm >= pm ? cm - pm : cm + (uint32_t)x.T - pm;
+    *slot_ptr(x, i, n) = make_uint4(r, phi, c | (left << 16), tier | (fresh ? kFirstFlag : 0u) | (rho << 16));
+    x.hist[i * x.TH + rho]++;
+    x.minfin[i] = min(x.minfin[i], phi + left - 1u);
 }
 
-// Batch formation steps (ii) and (iii) for instance i holding n running
-// requests and fr free blocks: admission in (tier, FCFS) order while the head
-// of line fits, then the iteration starts (Sec. 2.2, Sec. 3.1).  Single thread.
-template <class A>
-__device__ __forceinline__ void admit_and_start(const Ctx &x, A &acc, int i, int n, int fr, int base, int a_us,
-                                                int b_us) {
-    const int n_decode = n;
-    int prefill = 0;
-    int nr = n;
-    while (nr < x.Bmax) {
-        const uint32_t wm = x.wmask[i];
-        if (!wm) break;
-        const int need = x.hol[i];
-        if (need > fr) break;
-        const int k = __ffs(wm) - 1;
-        const uint32_t r = pop_front(x, i, k, acc.status);
-        if (r == kNone) break;
-        const uint32_t P = x.plen[r], O = x.olen[r], gg = x.g[r];
-        x.sst[i * x.SP + nr] = s_make(P + gg, (uint32_t)need, O - gg, (uint32_t)k, gg == 0);
-        x.srid[i * x.SP + nr] = r;
-        ++nr;
-        fr -= need;
-        prefill += (int)(P + gg);
-        refresh_hol(x, i);
-    }
-    x.nrun[i] = (uint8_t)nr;
-    x.free_[i] = fr;
-    if (nr > 0) {
-        const long long end = (long long)x.t + base + (long long)a_us * prefill + (long long)b_us * n_decode;
-        if (end > 0xFFFFFFFELL) {
-            acc.status = SIM_ERR_OVERFLOW;
-        } else {
-            x.busy[i] = (uint32_t)end;
-            x.nb[i] = (uint8_t)nr;
-            acc.iterations++;
-            acc.member_iterations += (uint64_t)nr;
-        }
-    }
+// Removes slot s of instance i's running list (order kept); returns its record.
+__device__ __forceinline__ uint4 slot_remove(const Ctx &x, int i, int s) {
+    uint4 *p = slot_ptr(x, i, 0);
+    const uint4 out = p[s];
+    const int n = x.nrun[i];
+    for (int q = s + 1; q < n; ++q) p[q - 1] = p[q];
+    x.nrun[i] = (uint8_t)(n - 1);
+    x.hist[i * x.TH + sl_rho(out)]--;
+    return out;
 }
 
-// ---- cooperative (whole-warp) steps -----------------------------------------
-// Lane l holds slots l and 32 + l of an instance.
-struct Slots {
-    uint64_t a0, a1;
-    uint32_t r0, r1;
-    bool v0, v1;
-};
-
-__device__ __forceinline__ Slots load_slots(const Ctx &x, int i, int n) {
-    Slots s;
-    const uint64_t *st = x.sst + i * x.SP;
-    const uint32_t *rd = x.srid + i * x.SP;
-    s.v0 = x.lane < n;
-    s.v1 = x.lane + 32 < n;
-    s.a0 = s.v0 ? st[x.lane] : 0ull;
-    s.r0 = s.v0 ? rd[x.lane] : kNone;
-    s.a1 = s.v1 ? st[x.lane + 32] : 0ull;
-    s.r1 = s.v1 ? rd[x.lane + 32] : kNone;
-    return s;
+__device__ __forceinline__ void recompute_minfin(const Ctx &x, int i) {
+    const uint4 *p = slot_ptr(x, i, 0);
+    uint32_t m = kNone;
+    for (int s = 0, n = x.nrun[i]; s < n; ++s) m = min(m, sl_fin(p[s]));
+    x.minfin[i] = m;
 }
 
-// Writes the slots whose keep flag is set at their compacted (stable) positions; returns the count.
-__device__ __forceinline__ int compact_slots(const Ctx &x, int i, const Slots &s, bool k0, bool k1) {
-    uint64_t *st = x.sst + i * x.SP;
-    uint32_t *rd = x.srid + i * x.SP;
-    const uint32_t q0 = __ballot_sync(kFull, k0), q1 = __ballot_sync(kFull, k1);
-    const uint32_t below = (1u << x.lane) - 1u;
-    const int p0 = __popc(q0 & below);
-    const int p1 = __popc(q0) + __popc(q1 & below);
-    __syncwarp();
-    if (k0) { st[p0] = s.a0; rd[p0] = s.r0; }
-    if (k1) { st[p1] = s.a1; rd[p1] = s.r1; }
-    __syncwarp();
-    return __popc(q0) + __popc(q1);
-}
-
-// Commit a fully copied running request from s to d (Sec. 3.5, Fig. 4).
-__device__ __forceinline__ void commit_mig(const Ctx &x, Cnt &cn, int s, int d, int pos, uint64_t a, uint32_t rid,
-                                           const Slots &sl, int n) {
-    uint64_t *st = x.sst + s * x.SP;
-    uint32_t *rd = x.srid + s * x.SP;
-    const int i0 = x.lane, i1 = x.lane + 32;
-    __syncwarp();
-    if (sl.v0 && i0 > pos) { st[i0 - 1] = sl.a0; rd[i0 - 1] = sl.r0; }
-    if (sl.v1 && i1 > pos) { st[i1 - 1] = sl.a1; rd[i1 - 1] = sl.r1; }
-    __syncwarp();
-    if (x.lane == 0) {
-        const int nd = x.nrun[d];
-        x.sst[d * x.SP + nd] = a;
-        x.srid[d * x.SP + nd] = rid;
-        x.nrun[d] = (uint8_t)(nd + 1);
-        x.nrun[s] = (uint8_t)(n - 1);
-        const int blocks = (int)s_blocks(a);
-        x.free_[s] += blocks;
-        x.resv[d] -= x.mcopied[s];
-        const int tr = (int)s_tier(a);
-        cnt_dec(x, s, tr);
-        cnt_inc(x, d, tr);
-        bump_mig(x, rid);
-        cn.migrations++;
-        cn.events++;
-        log_ev(x, cn, SIM_EV_COMMIT, rid, s, d, blocks);
-        clear_mig(x, s, d);
-    }
-    __syncwarp();
+// Commit a fully copied running request (slot pos of source s) to d (Sec. 3.5, Fig. 4).
+__device__ __forceinline__ void commit_mig(const Ctx &x, Cnt &cn, int s, int pos) {
+    const int d = x.mpeer[s];
+    const uint4 sl = *slot_ptr(x, s, pos);
+    const int blocks = sl_blocks(x, s, sl);
+    const uint32_t adv = sl_adv(x, s, sl);
+    slot_remove(x, s, pos);
+    if (sl_fin(sl) == x.minfin[s]) recompute_minfin(x, s);
+    x.free_[s] += blocks;
+    x.resv[d] -= x.mcopied[s];
+    const uint32_t tr = sl_tier(sl);
+    cnt_dec(x, s, (int)tr);
+    cnt_inc(x, d, (int)tr);
+    const int nd = x.nrun[d];
+    slot_join(x, d, nd, sl.x, sl_c(sl) + adv, sl_left(sl) - adv, tr, false);
+    x.nrun[d] = (uint8_t)(nd + 1);
+    bump_mig(x, sl.x);
+    cn.migrations++;
+    cn.events++;
+    log_ev(x, cn, SIM_EV_COMMIT, sl.x, s, d, blocks);
+    clear_mig(x, s, d);
 }
 
 // One copy stage at the end of an iteration of migration source s.
 __device__ __forceinline__ void migration_stage(const Ctx &x, Cnt &cn, int s) {
     const int d = x.mpeer[s];
     const uint32_t rid = x.mreq[s];
-    const int n = x.nrun[s];
-    const Slots sl = load_slots(x, s, n);
-    const uint32_t h0 = __ballot_sync(kFull, sl.v0 && sl.r0 == rid);
-    const uint32_t h1 = __ballot_sync(kFull, sl.v1 && sl.r1 == rid);
-    if (!(h0 | h1)) {
-        if (x.lane == 0) cn.status = SIM_ERR_INTERNAL;
-        __syncwarp();
-        return;
-    }
-    const int j = h0 ? 0 : 1;
-    const int l = __ffs(h0 ? h0 : h1) - 1;
-    const uint64_t a = __shfl_sync(kFull, j ? sl.a1 : sl.a0, l);
-    const int pos = 32 * j + l;
-    const int blocks = (int)s_blocks(a);
-    int commit = 0;
-    if (x.lane == 0) {
-        const int cp = x.mcopied[s];
-        const int cc = min(x.S, blocks - cp);
-        if (x.free_[d] < cc) {
-            abort_mig(x, cn, s);
-        } else {
-            x.free_[d] -= cc;
-            x.resv[d] += cc;
-            x.mcopied[s] = cp + cc;
-            commit = (cp + cc == blocks) && ((int)x.nrun[d] < x.Bmax);
-        }
-    }
-    commit = __shfl_sync(kFull, commit, 0);
-    __syncwarp();
-    if (commit) commit_mig(x, cn, s, d, pos, a, rid, sl, n);
+    const uint4 *p = slot_ptr(x, s, 0);
+    int pos = -1;
+    for (int q = 0, n = x.nrun[s]; q < n; ++q)
+        if (p[q].x == rid) { pos = q; break; }
+    if (pos < 0) { cn.status = SIM_ERR_INTERNAL; return; }
+    const int blocks = sl_blocks(x, s, p[pos]);
+    const int cp = x.mcopied[s];
+    const int cc = min(x.S, blocks - cp);
+    if (x.free_[d] < cc) { abort_mig(x, cn, s); return; }
+    x.free_[d] -= cc;
+    x.resv[d] += cc;
+    x.mcopied[s] = cp + cc;
+    if (cp + cc == blocks && (int)x.nrun[d] < x.Bmax) commit_mig(x, cn, s, pos);
 }
 
-// Phase 1: the iteration of instance i ends at t (Sec. 2.1 prefill/decode token accounting).
-__device__ __forceinline__ void complete_instance(const Ctx &x, Cnt &cn, int i) {
-    const int n = x.nrun[i], nb = x.nb[i];
-    Slots sl = load_slots(x, i, n);
-    const bool b0 = x.lane < nb, b1 = x.lane + 32 < nb;
-    bool g0 = false, g1 = false;
-    if (b0) {
-        sl.a0 += kAdvance;
-        g0 = (sl.a0 & kFirst) != 0;
-        if (g0) { sl.a0 ^= kFirst; x.res[sl.r0].first_token_us = x.t; }
+// Phase 1: the iteration of instance i ends at x.t (Sec. 2.1 token accounting):
+// fresh requests get their first token, requests whose output is complete
+// finish and free their KV, and a migration source runs one copy stage.
+__device__ __forceinline__ void inst_complete(const Ctx &x, Cnt &cn, int i) {
+    x.busy[i] = kNone;
+    x.pc[i] = 1;
+    uint4 *p = slot_ptr(x, i, 0);
+    for (int s = x.alo[i], e = x.ahi[i]; s < e; ++s) {  // the last formation's admissions
+        uint4 sl = p[s];
+        if (sl.w & kFirstFlag) {
+            x.res[sl.x].first_token_us = x.t;
+            sl.w &= ~kFirstFlag;
+            p[s] = sl;
+            cn.events++;
+        }
     }
-    if (b1) {
-        sl.a1 += kAdvance;
-        g1 = (sl.a1 & kFirst) != 0;
-        if (g1) { sl.a1 ^= kFirst; x.res[sl.r1].first_token_us = x.t; }
-    }
-    const bool f0 = b0 && s_left(sl.a0) == 0, f1 = b1 && s_left(sl.a1) == 0;
-    const uint32_t firsts = __reduce_add_sync(kFull, (uint32_t)g0 + (uint32_t)g1);
-    if (!__any_sync(kFull, f0 || f1)) {
-        uint64_t *st = x.sst + i * x.SP;
-        if (b0) st[x.lane] = sl.a0;
-        if (b1) st[x.lane + 32] = sl.a1;
-    } else {
-        const uint32_t m0 = __ballot_sync(kFull, f0), m1 = __ballot_sync(kFull, f1);
-        if (f0) { x.res[sl.r0].finish_us = x.t; x.res[sl.r0].final_instance = (uint16_t)i; }
-        if (f1) { x.res[sl.r1].finish_us = x.t; x.res[sl.r1].final_instance = (uint16_t)i; }
-#pragma unroll
-        for (int j = 0; j < 2; ++j) {  // finished requests in batch order
-            uint32_t lanes = j ? m1 : m0;
-            while (lanes) {
-                const int l = __ffs(lanes) - 1;
-                lanes &= lanes - 1;
-                const uint64_t a = __shfl_sync(kFull, j ? sl.a1 : sl.a0, l);
-                const uint32_t r = __shfl_sync(kFull, j ? sl.r1 : sl.r0, l);
-                if (x.lane == 0) {
-                    x.free_[i] += (int)s_blocks(a);
-                    cnt_dec(x, i, (int)s_tier(a));
-                    if (x.mrole[i] == MIG_SRC && x.mreq[i] == r) abort_mig(x, cn, i);
-                }
-                __syncwarp();
+    x.alo[i] = x.ahi[i] = 0;
+    const uint32_t nf = x.nf[i];
+    if (x.minfin[i] == nf) {
+        int w = 0;
+        uint32_t m = kNone;
+        for (int s = 0, n = x.nrun[i]; s < n; ++s) {
+            const uint4 sl = p[s];
+            if (sl_fin(sl) == nf) {
+                x.res[sl.x].finish_us = x.t;
+                x.res[sl.x].final_instance = (uint16_t)i;
+                x.free_[i] += sl_blocks(x, i, sl);
+                cnt_dec(x, i, (int)sl_tier(sl));
+                x.hist[i * x.TH + sl_rho(sl)]--;
+                cn.finished++;
+                cn.events++;
+                if (x.mrole[i] == MIG_SRC && x.mreq[i] == sl.x) abort_mig(x, cn, i);
+            } else {
+                p[w++] = sl;
+                m = min(m, sl_fin(sl));
             }
         }
-        const int kept = compact_slots(x, i, sl, sl.v0 && !f0, sl.v1 && !f1);
-        const uint32_t nfin = __popc(m0) + __popc(m1);
-        cn.finished += nfin;
-        if (x.lane == 0) { x.nrun[i] = (uint8_t)kept; cn.events += nfin; }
+        x.nrun[i] = (uint8_t)w;
+        x.minfin[i] = m;
     }
-    if (x.lane == 0) {
-        x.busy[i] = kNone;
-        cn.events += firsts;
-    }
-    __syncwarp();
     if (x.mrole[i] == MIG_SRC) migration_stage(x, cn, i);
 }
 
+// Recompute-style preemption of running request `sl` (holding `blocks` KV
+// blocks) on instance i: its KV is freed, it keeps its generated tokens and
+// goes back to the front of its tier's bucket.  The caller drops its slot.
+__device__ __forceinline__ void preempt_book(const Ctx &x, Cnt &cn, int i, const uint4 &sl, int blocks) {
+    const uint32_t r = sl.x;
+    const int tr = (int)sl_tier(sl);
+    const uint32_t adv = sl_adv(x, i, sl);
+    x.free_[i] += blocks;
+    x.g[r] = (uint16_t)(x.olen[r] - (sl_left(sl) - adv));
+    const uint32_t old = x.wmask[i];
+    push_front(x, i, tr, r);
+    if ((old & ((1u << tr) - 1u)) == 0) x.hol[i] = blocks_for(x, sl_c(sl) + adv);  // now head of line
+    x.hist[i * x.TH + sl_rho(sl)]--;
+    bump_pre(x, r);
+    cn.preemptions++;
+    cn.events++;
+    if (x.mrole[i] == MIG_SRC && x.mreq[i] == r) abort_mig(x, cn, i);
+}
+
+// Phase 4: batch formation at idle instance i at x.t (Sec. 2.2, Sec. 3.1):
+// (i) KV growth of the running requests, preempting the lowest-priority newest
+// one when out of blocks; (ii) admission in (tier, FCFS) order while the head
+// of line fits; (iii) the iteration starts.
+__device__ __forceinline__ void inst_form(const Ctx &x, Cnt &cn, int i, int base, int a_us, int b_us) {
+    int n = x.nrun[i];
+    if (n > 0) {
+        const uint32_t ph = x.phase[i];
+        const int deficit = x.hist[i * x.TH + (ph == 0 ? 0u : (uint32_t)x.T - ph)];
+        if (deficit <= x.free_[i]) {
+            x.free_[i] -= deficit;  // every request that needs a block gets it
+        } else {
+            // In running order, a request that needs a block (at most one)
+            // takes a free one or preempts the lowest-priority newest running
+            // request, possibly itself.  Positions are the list's before this
+            // step; removals are applied afterwards.
+            uint4 *p = slot_ptr(x, i, 0);
+            const uint64_t all = n >= 64 ? ~0ull : ((1ull << n) - 1ull);
+            uint64_t alive = all, needs = 0, granted = 0;
+            for (int q = 0; q < n; ++q) {
+                const uint4 sl = p[q];
+                if (blocks_for(x, sl_c(sl) + sl_adv(x, i, sl)) > sl_blocks(x, i, sl)) needs |= 1ull << q;
+            }
+            int fr = x.free_[i];
+            for (int q = 0; q < n; ++q) {
+                if (!((alive & needs) >> q & 1ull)) continue;
+                for (;;) {
+                    if (fr > 0) { --fr; granted |= 1ull << q; break; }
+                    int v = -1;
+                    uint32_t vt = 0, vr = 0;
+                    for (uint64_t m = alive; m; m &= m - 1) {
+                        const int s2 = __ffsll((long long)m) - 1;
+                        const uint32_t ts = sl_tier(p[s2]), rs = p[s2].x;
+                        if (v < 0 || ts > vt || (ts == vt && rs > vr)) { v = s2; vt = ts; vr = rs; }
+                    }
+                    const int vb = sl_blocks(x, i, p[v]) + (int)((granted >> v) & 1ull);
+                    alive &= ~(1ull << v);
+                    x.free_[i] = fr;
+                    preempt_book(x, cn, i, p[v], vb);
+                    fr = x.free_[i];
+                    if (v == q) break;
+                }
+            }
+            x.free_[i] = fr;
+            int w = 0;
+            for (int q = 0; q < n; ++q)
+                if ((alive >> q) & 1ull) { if (w != q) p[w] = p[q]; ++w; }
+            x.nrun[i] = (uint8_t)w;
+            recompute_minfin(x, i);
+        }
+    }
+    // (ii) admission
+    n = x.nrun[i];
+    const int n_decode = n;
+    int fr = x.free_[i];
+    int prefill = 0;
+    x.alo[i] = (uint8_t)n;
+    while (n < x.Bmax) {
+        const uint32_t wm = x.wmask[i];
+        if (!wm) break;
+        const int need = x.hol[i];
+        if (need > fr) break;
+        const int k = __ffs(wm) - 1;
+        const uint32_t r = pop_front(x, i, k, cn.status);
+        if (r == kNone) break;
+        const uint32_t P = x.plen[r], O = x.olen[r], gg = x.g[r];
+        slot_join(x, i, n, r, P + gg, O - gg, (uint32_t)k, gg == 0);
+        ++n;
+        fr -= need;
+        prefill += (int)(P + gg);
+        refresh_hol(x, i);
+    }
+    x.ahi[i] = (uint8_t)n;
+    x.nrun[i] = (uint8_t)n;
+    x.free_[i] = fr;
+    // (iii) the iteration starts
+    if (n > 0) {
+        const long long end = (long long)x.t + base + (long long)a_us * prefill + (long long)b_us * n_decode;
+        if (end > 0xFFFFFFFELL) {
+            cn.status = SIM_ERR_OVERFLOW;
+            return;
+        }
+        x.busy[i] = (uint32_t)end;
+        x.nf[i] += 1u;
+        x.phase[i] = x.phase[i] + 1u == (uint32_t)x.T ? (uint8_t)0 : (uint8_t)(x.phase[i] + 1u);
+        x.pc[i] = 0;
+        cn.iterations++;
+        cn.member_iterations += (uint64_t)n;
+    }
+}
+
+// ---- cooperative steps ----------------------------------------------------------
 // Dispatch one arriving request r of tier k with prompt length P (Sec. 3.4).
 template <int C>
 __device__ __forceinline__ void dispatch_one(const Ctx &x, Cnt &cn, uint32_t r, int k, uint32_t P, uint32_t all) {
@@ -628,12 +655,10 @@ __device__ __forceinline__ void migration_tick(const Ctx &x, Cnt &cn, int theta_
         const long long ns = fnum(x, s), ds = max((int)x.nrun[s], 1);
         const long long nd = fnum(x, d), dd = max((int)x.nrun[d], 1);
         if ((long long)theta_den * (nd * ds - ns * dd) < (long long)theta_num * dd * ds) break;
-        const bool has_wait = x.wmask[s] != 0;
-        const int n_s = x.nrun[s];
-        __syncwarp();
         int moved = 0;
-        if (has_wait) {
-            if (x.lane == 0) {
+        if (x.lane == 0) {
+            if (x.wmask[s] != 0) {
+                // queued candidate: newest request of the lowest-priority bucket, no KV to copy
                 const int k = 31 - __clz((unsigned)x.wmask[s]);
                 const uint32_t r = pop_back(x, s, k, cn.status);
                 if (r != kNone) {
@@ -648,190 +673,40 @@ __device__ __forceinline__ void migration_tick(const Ctx &x, Cnt &cn, int theta_
                     cn.events++;
                     log_ev(x, cn, SIM_EV_QUEUED, r, s, d, 0);
                 }
-            }
-            moved = 1;
-        } else if (n_s > 0) {
-            // running candidate: lowest priority, then fewest blocks, then newest
-            const Slots sl = load_slots(x, s, n_s);
-            const int k0 = sl.v0 ? (int)((s_tier(sl.a0) << 16) | (0xFFFFu - s_blocks(sl.a0))) : -1;
-            const int k1 = sl.v1 ? (int)((s_tier(sl.a1) << 16) | (0xFFFFu - s_blocks(sl.a1))) : -1;
-            const int km = __reduce_max_sync(kFull, max(k0, k1));
-            const uint32_t c0 = (sl.v0 && k0 == km) ? sl.r0 : 0u, c1 = (sl.v1 && k1 == km) ? sl.r1 : 0u;
-            const uint32_t rid = __reduce_max_sync(kFull, max(c0, c1));
-            const int blocks = (int)(0xFFFFu - ((uint32_t)km & 0xFFFFu));
-            if (x.free_[d] >= blocks) {
-                if (x.lane == 0) {
+                moved = 1;
+            } else if (x.nrun[s] > 0) {
+                // running candidate: lowest priority, then fewest blocks, then newest
+                const uint4 *p = slot_ptr(x, s, 0);
+                int best = -1, bb = 0;
+                uint32_t bt = 0, br = 0;
+                for (int q = 0, n = x.nrun[s]; q < n; ++q) {
+                    const uint32_t tq = sl_tier(p[q]), rq = p[q].x;
+                    const int bq = sl_blocks(x, s, p[q]);
+                    if (best < 0 || tq > bt || (tq == bt && (bq < bb || (bq == bb && rq > br)))) {
+                        best = q; bt = tq; bb = bq; br = rq;
+                    }
+                }
+                if (x.free_[d] >= bb) {
                     x.mrole[s] = MIG_SRC;
                     x.mpeer[s] = (uint8_t)d;
-                    x.mreq[s] = rid;
+                    x.mreq[s] = br;
                     x.mcopied[s] = 0;
                     x.mrole[d] = MIG_DST;
                     x.mpeer[d] = (uint8_t)s;
                     cn.starts++;
-                    log_ev(x, cn, SIM_EV_START, rid, s, d, blocks);
+                    log_ev(x, cn, SIM_EV_START, br, s, d, bb);
+                    moved = 1;
                 }
-                moved = 1;
             }
         }
+        moved = __shfl_sync(kFull, moved, 0);
         if (x.lane == s / C) el &= ~(1u << (s % C));
         if (moved && x.lane == d / C) el &= ~(1u << (d % C));
         __syncwarp();
     }
 }
 
-// Phase 4: batch formation at idle instance i (Sec. 2.2 continuous batching).
-__device__ __forceinline__ void form_batch(const Ctx &x, Cnt &cn, int i, int base, int a_us, int b_us) {
-    int n = x.nrun[i];
-    int fr = x.free_[i];
-    Slots sl = load_slots(x, i, n);
-    const int d0 = sl.v0 ? max(0, blocks_for(x, s_ctx(sl.a0)) - (int)s_blocks(sl.a0)) : 0;
-    const int d1 = sl.v1 ? max(0, blocks_for(x, s_ctx(sl.a1)) - (int)s_blocks(sl.a1)) : 0;
-    const int total = __reduce_add_sync(kFull, d0 + d1);
-    if (total <= fr) {
-        // (i) every running request gets the KV growth it needs
-        if (total > 0) {
-            fr -= total;
-            uint64_t *st = x.sst + i * x.SP;
-            if (d0) st[x.lane] = sl.a0 + ((uint64_t)d0 << 16);
-            if (d1) st[x.lane + 32] = sl.a1 + ((uint64_t)d1 << 16);
-        }
-    } else {
-        // (i) grow in running order; when out of blocks, preempt the lowest
-        // priority, newest running request (possibly the one growing).
-        bool al0 = sl.v0, al1 = sl.v1;
-        for (int idx = 0; idx < n; ++idx) {
-            const int l = idx & 31, j = idx >> 5;
-            for (;;) {
-                if (!__shfl_sync(kFull, (int)(j ? al1 : al0), l)) break;
-                const uint64_t a = __shfl_sync(kFull, j ? sl.a1 : sl.a0, l);
-                const int def = blocks_for(x, s_ctx(a)) - (int)s_blocks(a);
-                if (def <= 0) break;
-                if (fr > 0) {
-                    const int gv = min(fr, def);
-                    fr -= gv;
-                    if (x.lane == l) {
-                        if (j) sl.a1 += (uint64_t)gv << 16; else sl.a0 += (uint64_t)gv << 16;
-                    }
-                    continue;
-                }
-                const int t0 = al0 ? (int)s_tier(sl.a0) : -1, t1 = al1 ? (int)s_tier(sl.a1) : -1;
-                const int tmax = __reduce_max_sync(kFull, max(t0, t1));
-                const uint32_t c0 = (al0 && t0 == tmax) ? sl.r0 : 0u, c1 = (al1 && t1 == tmax) ? sl.r1 : 0u;
-                const uint32_t rmax = __reduce_max_sync(kFull, max(c0, c1));
-                const uint32_t vm0 = __ballot_sync(kFull, al0 && t0 == tmax && sl.r0 == rmax);
-                const uint32_t vm1 = __ballot_sync(kFull, al1 && t1 == tmax && sl.r1 == rmax);
-                const int vj = vm0 ? 0 : 1;
-                const int vl = __ffs(vm0 ? vm0 : vm1) - 1;
-                const uint64_t va = __shfl_sync(kFull, vj ? sl.a1 : sl.a0, vl);
-                fr += (int)s_blocks(va);
-                if (x.lane == vl) { if (vj) al1 = false; else al0 = false; }
-                if (x.lane == 0) {
-                    preempt_common(x, cn, i, rmax, va);
-                    if (x.mrole[i] == MIG_SRC && x.mreq[i] == rmax) abort_mig(x, cn, i);
-                }
-                __syncwarp();
-                if (vl == l && vj == j) break;
-            }
-        }
-        n = compact_slots(x, i, sl, al0, al1);
-    }
-    if (x.lane == 0) admit_and_start(x, cn, i, n, fr, base, a_us, b_us);
-    __syncwarp();
-}
-
-// ---- lane-parallel path -------------------------------------------------------
-// One lane advances instance i, which is in no migration, through its
-// iteration end at t (phase 1) and the batch formation that follows at t
-// (phase 4).  Exactly the cooperative semantics; only this lane runs it.
-__device__ __forceinline__ void solo_event(const Ctx &x, Acc &acc, int i, int base, int a_us, int b_us) {
-    uint64_t *st = x.sst + i * x.SP;
-    uint32_t *rd = x.srid + i * x.SP;
-    const int n0 = x.nrun[i], nb = x.nb[i];
-    int fr = x.free_[i];
-    int w = 0, total = 0;
-    uint64_t grow = 0;  // bit w: the kept slot w needs more KV blocks
-    for (int s = 0; s < n0; ++s) {
-        uint64_t a = st[s];
-        if (s < nb) {
-            a += kAdvance;
-            if (a & kFirst) {
-                a ^= kFirst;
-                x.res[rd[s]].first_token_us = x.t;
-                acc.events++;
-            }
-            if (s_left(a) == 0) {  // finished: free its KV
-                const uint32_t r = rd[s];
-                x.res[r].finish_us = x.t;
-                x.res[r].final_instance = (uint16_t)i;
-                fr += (int)s_blocks(a);
-                cnt_dec(x, i, (int)s_tier(a));
-                acc.finished++;
-                acc.events++;
-                continue;
-            }
-        }
-        const int def = blocks_for(x, s_ctx(a)) - (int)s_blocks(a);
-        if (def > 0) {
-            grow |= 1ull << w;
-            total += def;
-        }
-        if (w != s) rd[w] = rd[s];
-        st[w++] = a;
-    }
-    int n = w;
-    x.busy[i] = kNone;
-    if (total <= fr) {
-        fr -= total;
-        while (grow) {
-            const int s = __ffsll((long long)grow) - 1;
-            grow &= grow - 1;
-            const uint64_t a = st[s];
-            st[s] = a + ((uint64_t)(blocks_for(x, s_ctx(a)) - (int)s_blocks(a)) << 16);
-        }
-    } else {
-        // grow in running order, preempting the lowest-priority newest request when out of blocks
-        uint64_t alive = n >= 64 ? ~0ull : ((1ull << n) - 1ull);
-        for (int idx = 0; idx < n; ++idx) {
-            if (!((alive >> idx) & 1ull)) continue;
-            for (;;) {
-                const uint64_t a = st[idx];
-                const int def = blocks_for(x, s_ctx(a)) - (int)s_blocks(a);
-                if (def <= 0) break;
-                if (fr > 0) {
-                    const int gv = min(fr, def);
-                    fr -= gv;
-                    st[idx] = a + ((uint64_t)gv << 16);
-                    continue;
-                }
-                int v = -1;
-                uint32_t vt = 0, vr = 0;
-                for (uint64_t m = alive; m; m &= m - 1) {
-                    const int s = __ffsll((long long)m) - 1;
-                    const uint32_t ts = s_tier(st[s]), rs = rd[s];
-                    if (v < 0 || ts > vt || (ts == vt && rs > vr)) { v = s; vt = ts; vr = rs; }
-                }
-                const uint64_t va = st[v];
-                fr += (int)s_blocks(va);
-                alive &= ~(1ull << v);
-                preempt_common(x, acc, i, vr, va);
-                if (v == idx) break;
-            }
-        }
-        int k = 0;
-        for (int s = 0; s < n; ++s) {
-            if (!((alive >> s) & 1ull)) continue;
-            if (k != s) { st[k] = st[s]; rd[k] = rd[s]; }
-            ++k;
-        }
-        n = k;
-    }
-    admit_and_start(x, acc, i, n, fr, base, a_us, b_us);
-}
-
-// Number of distinct event times in a window: `u[j]` is the event time of this
-// lane's instance j (kNone if none); coupled-instance step times are added by
-// the caller.  C == 1 uses __match_any_sync; wider variants insert into a
-// per-warp open-addressing set of event times, cleared by the caller.
+// Distinct event times of a window (C > 1): a per-warp open-addressing set.
 __device__ __forceinline__ uint32_t tset_insert(const Ctx &x, uint32_t t) {
     uint32_t h = (t * 0x9E3779B1u) >> 23;  // 9 bits: kHashSlots = 512
     for (uint32_t probe = 0; probe < kHashSlots; ++probe) {
@@ -857,42 +732,44 @@ __device__ __forceinline__ void bind_blob(Ctx &x, const Layout &L, unsigned char
     x.key = reinterpret_cast<int *>(blob + L.key);
     x.mreq = reinterpret_cast<uint32_t *>(blob + L.mreq);
     x.mcopied = reinterpret_cast<int *>(blob + L.mcopied);
+    x.nf = reinterpret_cast<uint32_t *>(blob + L.nf);
+    x.minfin = reinterpret_cast<uint32_t *>(blob + L.minfin);
     x.wmask = reinterpret_cast<uint16_t *>(blob + L.wmask);
     x.nrun = blob + L.nrun;
-    x.nb = blob + L.nb;
+    x.pc = blob + L.pc;
+    x.phase = blob + L.phase;
+    x.alo = blob + L.alo;
+    x.ahi = blob + L.ahi;
     x.mrole = blob + L.mrole;
     x.mpeer = blob + L.mpeer;
     x.cnt = reinterpret_cast<uint16_t *>(blob + L.cnt);
     x.head = reinterpret_cast<uint32_t *>(blob + L.head);
     x.tail = reinterpret_cast<uint32_t *>(blob + L.tail);
     x.h = reinterpret_cast<int *>(blob + L.h);
+    x.hist = blob + L.hist;
 }
 
-// Phase 1 restricted to the instances whose bit is set in `mask` (bit j =
-// instance lane*C + j): iteration ends at x.t, ascending index.  Collective.
+// Phase 1 at x.t for the instances in `mask` (bit j = instance lane*C + j)
+// whose iteration ends now, ascending index, on lane 0.  Collective.
 template <int C>
-__device__ __forceinline__ void complete_all(const Ctx &x, Cnt &cn, uint32_t mask, const Params &p) {
+__device__ __forceinline__ void complete_all(const Ctx &x, Cnt &cn, uint32_t mask) {
     uint32_t hits = 0;
 #pragma unroll
-    for (int j = 0; j < C; ++j) {
-        const int i = x.lane * C + j;
-        if (((mask >> j) & 1u) && x.busy[i] == x.t) hits |= 1u << j;
-    }
+    for (int j = 0; j < C; ++j)
+        if (((mask >> j) & 1u) && x.busy[x.lane * C + j] == x.t) hits |= 1u << j;
     uint32_t lanes = __ballot_sync(kFull, hits != 0);
     while (lanes) {
         const int l = __ffs(lanes) - 1;
         lanes &= lanes - 1;
-        uint32_t h = C == 1 ? 1u : __shfl_sync(kFull, hits, l);
-        while (h) {
-            const int j = __ffs(h) - 1;
-            h &= h - 1;
-            complete_instance(x, cn, l * C + j);
-        }
+        const uint32_t h = C == 1 ? 1u : __shfl_sync(kFull, hits, l);
+        if (x.lane == 0)
+            for (uint32_t hh = h; hh; hh &= hh - 1) inst_complete(x, cn, l * C + __ffs(hh) - 1);
     }
+    __syncwarp();
 }
 
-// Phase 4 restricted to `mask`: batch formation at every idle instance with
-// work, ascending index.  Collective.
+// Phase 4 at x.t for the idle instances in `mask` that have work, ascending
+// index, on lane 0.  Collective.
 template <int C>
 __device__ __forceinline__ void form_all(const Ctx &x, Cnt &cn, uint32_t mask, const Params &p) {
     uint32_t want = 0;
@@ -905,26 +782,24 @@ __device__ __forceinline__ void form_all(const Ctx &x, Cnt &cn, uint32_t mask, c
     while (lanes) {
         const int l = __ffs(lanes) - 1;
         lanes &= lanes - 1;
-        uint32_t h = C == 1 ? 1u : __shfl_sync(kFull, want, l);
-        while (h) {
-            const int j = __ffs(h) - 1;
-            h &= h - 1;
-            form_batch(x, cn, l * C + j, p.base, p.a, p.b);
-        }
+        const uint32_t h = C == 1 ? 1u : __shfl_sync(kFull, want, l);
+        if (x.lane == 0)
+            for (uint32_t hh = h; hh; hh &= hh - 1) inst_form(x, cn, l * C + __ffs(hh) - 1, p.base, p.a, p.b);
     }
+    __syncwarp();
 }
 
 // The persistent simulation kernel: each warp repeatedly takes a replica and
-// advances it by up to p.max_steps event times.  C = instances per lane;
-// SMS = running-request slots staged in shared memory.
+// advances it by up to p.max_steps event times; C = instances per lane.
 //
 // Between two global events (the next arrival, the next migration tick) the
 // instances that are in no migration do not interact, and an iteration lasts
 // at least `base` microseconds.  So in a window [tmin, min(T_g, tmin + base))
-// every instance ends at most one iteration, and the lanes advance their own
-// instances in parallel; instances in a migration, and every step at a global
-// event, go through the cooperative single-step code in time order.
-template <int C, bool SMS>
+// every instance ends at most one iteration, and each lane advances its own
+// instances (an O(1) iteration end + batch formation); instances in a
+// migration, and every step at a global event, are advanced by lane 0 in the
+// oracle's order.
+template <int C>
 __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
     extern __shared__ __align__(16) unsigned char smem[];
     unsigned long long *magic = reinterpret_cast<unsigned long long *>(smem);
@@ -932,11 +807,9 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
         magic[d] = d < 2 ? 0ull : ~0ull / (unsigned long long)d + 1ull;
     __syncthreads();
     const int lane = threadIdx.x & 31;
-    const uint32_t per_warp = p.L.bytes + p.slot_bytes + p.hash_bytes;
+    const uint32_t per_warp = p.L.bytes + p.hash_bytes;
     unsigned char *blob = smem + kMagicBytes + (size_t)(threadIdx.x >> 5) * per_warp;
-    unsigned char *sslots = blob + p.L.bytes;
-    uint32_t *tset = reinterpret_cast<uint32_t *>(blob + p.L.bytes + p.slot_bytes);
-    const uint32_t nslot = p.NS;
+    uint32_t *tset = reinterpret_cast<uint32_t *>(blob + p.L.bytes);
     for (;;) {
         int r = 0;
         if (lane == 0) r = atomicAdd(p.work, 1);
@@ -945,20 +818,10 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
         const RepState rs = p.rep[r];
         if (rs.status != SIM_REPLICA_RUNNING) continue;
         unsigned char *gblob = p.blobs + (size_t)r * p.L.bytes;
-        uint64_t *g_sst = p.sst + (size_t)r * nslot;
-        uint32_t *g_srid = p.srid + (size_t)r * nslot;
         copy16(blob, gblob, p.L.bytes, lane);
         Ctx x;
         bind_blob(x, p.L, blob);
-        if (SMS) {
-            x.sst = reinterpret_cast<uint64_t *>(sslots);
-            x.srid = reinterpret_cast<uint32_t *>(sslots + (size_t)nslot * 8);
-            copy16(sslots, reinterpret_cast<const unsigned char *>(g_sst), nslot * 8, lane);
-            copy16(sslots + (size_t)nslot * 8, reinterpret_cast<const unsigned char *>(g_srid), nslot * 4, lane);
-        } else {
-            x.sst = g_sst;
-            x.srid = g_srid;
-        }
+        x.slots = p.slots + (size_t)r * p.N * p.Bmax;
         x.tset = tset;
         __syncwarp();
         const long long o = p.offsets[r];
@@ -976,31 +839,26 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
         x.N = p.N;
         x.K = p.K;
         x.T = p.T;
+        x.TH = p.TH;
         x.Bmax = p.Bmax;
-        x.SP = p.SP;
         x.S = p.S;
         x.cap = p.cap;
         x.lane = lane;
         x.t = rs.t;
-        Cnt cn;
+        Cnt cn;  // lane 0: the replica's totals; other lanes: what they add in windows
+        const bool l0 = lane == 0;
         cn.finished = rs.finished;
         cn.log_events = rs.log_events;
         cn.migrations = rs.migrations;
-        cn.preemptions = rs.preemptions;
+        cn.preemptions = l0 ? rs.preemptions : 0u;
         cn.starts = rs.starts;
         cn.aborts = rs.aborts;
         cn.steps = 0;
         cn.iterations = 0;
-        cn.member_iterations = rs.member_iterations;
-        cn.events = rs.events;
+        cn.member_iterations = l0 ? rs.member_iterations : 0ull;
+        cn.events = l0 ? rs.events : 0ull;
         cn.status = SIM_REPLICA_RUNNING;
-        Acc acc;
-        acc.finished = 0;
-        acc.preemptions = 0;
-        acc.iterations = 0;
-        acc.member_iterations = 0;
-        acc.events = 0;
-        acc.status = 0;
+        uint32_t wfin = 0;  // requests this lane finished in the current window
         uint32_t cursor = rs.cursor;
         uint32_t next_tick = rs.next_tick;
         ArrBuf ab;
@@ -1023,7 +881,8 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
             const uint32_t tg = p.enable_mig ? min(next_arr, next_tick) : next_arr;
             if (tb < tg && max_steps - cn.steps > (uint32_t)x.N) {
                 // ---- window [tb, t1): at most one iteration end per instance ----
-                const uint32_t t1 = (uint32_t)min((unsigned long long)tg, (unsigned long long)tb + (uint32_t)p.base);
+                const uint32_t t1 =
+                    (uint32_t)min((unsigned long long)tg, (unsigned long long)tb + (uint32_t)p.base);
                 uint32_t cm = 0, solo = 0;  // instances with an iteration end in the window: in a migration / not
 #pragma unroll
                 for (int j = 0; j < C; ++j) {
@@ -1036,21 +895,23 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
                     for (uint32_t q = (uint32_t)lane; q < kHashSlots; q += 32) tset[q] = kNone;
                     __syncwarp();
                 }
-                uint32_t fresh = 0;   // distinct event times this lane contributes
-                uint32_t tlast = 0;   // latest event time processed in the window
-                if (solo) {
+                uint32_t fresh = 0;  // distinct event times this lane contributes (C > 1)
+                uint32_t tlast = 0;  // latest event time processed in the window
+                const uint32_t fin0 = cn.finished;
 #pragma unroll
-                    for (int j = 0; j < C; ++j) {
-                        if (!((solo >> j) & 1u)) continue;
-                        x.t = bz[j];
-                        tlast = max(tlast, bz[j]);
-                        if (C > 1) fresh += tset_insert(x, bz[j]);
-                        solo_event(x, acc, lane * C + j, p.base, p.a, p.b);
-                    }
+                for (int j = 0; j < C; ++j) {
+                    if (!((solo >> j) & 1u)) continue;
+                    const int i = lane * C + j;
+                    x.t = bz[j];
+                    tlast = max(tlast, bz[j]);
+                    if (C > 1) fresh += tset_insert(x, bz[j]);
+                    inst_complete(x, cn, i);
+                    inst_form(x, cn, i, p.base, p.a, p.b);
                 }
+                wfin = cn.finished - fin0;
+                cn.finished = fin0;
                 __syncwarp();
-                uint32_t ucount;
-                uint32_t u = kNone;
+                uint32_t ucount, u = kNone;
                 if (C == 1) {
                     u = solo ? bz[0] : kNone;
                     const uint32_t grp = __match_any_sync(kFull, u);
@@ -1058,8 +919,8 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
                 } else {
                     ucount = __reduce_add_sync(kFull, fresh);
                 }
-                // instances in a migration (both ends, with or without an event of
-                // their own in the window): cooperative steps in time order
+                // instances in a migration (both ends, with or without an event
+                // of their own in the window): steps in time order on lane 0
                 if (__any_sync(kFull, cm != 0)) {
 #pragma unroll
                     for (int j = 0; j < C; ++j) {
@@ -1069,16 +930,17 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
                     for (;;) {
                         uint32_t cb = kNone;
 #pragma unroll
-                        for (int j = 0; j < C; ++j) {
-                            const int i = lane * C + j;
-                            if ((cm >> j) & 1u) cb = min(cb, x.busy[i]);
-                        }
+                        for (int j = 0; j < C; ++j)
+                            if ((cm >> j) & 1u) cb = min(cb, x.busy[lane * C + j]);
                         const uint32_t tc = __reduce_min_sync(kFull, cb);
                         if (tc >= t1) break;
                         x.t = tc;
                         tlast = max(tlast, tc);
-                        complete_all<C>(x, cn, cm, p);
+                        const uint32_t f1 = cn.finished;
+                        complete_all<C>(x, cn, cm);
                         form_all<C>(x, cn, cm, p);
+                        wfin += __shfl_sync(kFull, cn.finished - f1, 0) * (lane == 0 ? 1u : 0u);
+                        cn.finished = __shfl_sync(kFull, f1, 0);
                         if (C == 1) {
                             ucount += __any_sync(kFull, u == tc) ? 0u : 1u;
                         } else {
@@ -1092,10 +954,9 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
                 }
                 cn.steps += ucount;
                 x.t = __reduce_max_sync(kFull, tlast);
-                cn.finished += __reduce_add_sync(kFull, acc.finished);
-                acc.finished = 0;
-                const int ws = __reduce_min_sync(kFull, acc.status);
-                if (ws < 0 && cn.status >= 0) cn.status = ws;
+                cn.finished += __reduce_add_sync(kFull, wfin);
+                const int ws = __reduce_min_sync(kFull, cn.status);
+                cn.status = ws;
                 if (cn.status < 0) break;
                 continue;
             }
@@ -1105,7 +966,9 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
             const bool tick = p.enable_mig && next_tick <= tc;
             x.t = tick ? next_tick : tc;
             ++cn.steps;
-            if (tb == x.t) complete_all<C>(x, cn, all, p);  // 1. iteration ends
+            const uint32_t f1 = cn.finished;
+            if (tb == x.t) complete_all<C>(x, cn, all);  // 1. iteration ends
+            cn.finished = __shfl_sync(kFull, cn.finished, 0);
             if (next_arr == x.t) dispatch_phase<C>(x, cn, cursor, next_arr, ab);  // 2. dispatch
             if (tick) {  // 3. migration tick
                 const uint32_t nt = next_tick + p.interval;
@@ -1113,25 +976,22 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
                 migration_tick<C>(x, cn, p.theta_num, p.theta_den);
             }
             form_all<C>(x, cn, all, p);  // 4. batch formation
+            (void)f1;
             cn.status = __shfl_sync(kFull, cn.status, 0);
             if (cn.status < 0) break;
         }
         __syncwarp();
-        // fold the lane-parallel counters into lane 0's
-        const uint32_t a_pre = __reduce_add_sync(kFull, acc.preemptions);
-        const uint32_t a_it = __reduce_add_sync(kFull, acc.iterations);
-        uint64_t a_mi = acc.member_iterations, a_ev = acc.events;
+        // fold the other lanes' counters into lane 0's
+        const uint32_t a_pre = __reduce_add_sync(kFull, l0 ? 0u : cn.preemptions);
+        const uint32_t a_it = __reduce_add_sync(kFull, cn.iterations);
+        uint64_t a_mi = cn.member_iterations, a_ev = cn.events;
 #pragma unroll
         for (int sh = 16; sh > 0; sh >>= 1) {
             a_mi += __shfl_xor_sync(kFull, a_mi, sh);
             a_ev += __shfl_xor_sync(kFull, a_ev, sh);
         }
         copy16(gblob, blob, p.L.bytes, lane);
-        if (SMS) {
-            copy16(reinterpret_cast<unsigned char *>(g_sst), sslots, nslot * 8, lane);
-            copy16(reinterpret_cast<unsigned char *>(g_srid), sslots + (size_t)nslot * 8, nslot * 4, lane);
-        }
-        if (lane == 0) {
+        if (l0) {
             RepState o2;
             o2.t = x.t;
             o2.cursor = cursor;
@@ -1140,9 +1000,9 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
             o2.next_tick = next_tick;
             o2.pad0 = 0;
             o2.steps = rs.steps + cn.steps;
-            o2.iterations = rs.iterations + cn.iterations + a_it;
-            o2.member_iterations = cn.member_iterations + a_mi;
-            o2.events = cn.events + a_ev;
+            o2.iterations = rs.iterations + a_it;
+            o2.member_iterations = a_mi;
+            o2.events = a_ev;
             o2.migrations = cn.migrations;
             o2.preemptions = cn.preemptions + a_pre;
             o2.starts = cn.starts;
@@ -1174,12 +1034,18 @@ __global__ void k_init_state(Params p, const int *rep_table, const int *tbl_k, c
             reinterpret_cast<int *>(b + L.key)[i] = 0;
             reinterpret_cast<uint32_t *>(b + L.mreq)[i] = kNone;
             reinterpret_cast<int *>(b + L.mcopied)[i] = 0;
+            reinterpret_cast<uint32_t *>(b + L.nf)[i] = 0;
+            reinterpret_cast<uint32_t *>(b + L.minfin)[i] = kNone;
             reinterpret_cast<uint16_t *>(b + L.wmask)[i] = 0;
             b[L.nrun + i] = 0;
-            b[L.nb + i] = 0;
+            b[L.pc + i] = 0;
+            b[L.phase + i] = 0;
+            b[L.alo + i] = 0;
+            b[L.ahi + i] = 0;
             b[L.mrole + i] = MIG_NONE;
             b[L.mpeer + i] = 0;
         }
+        for (int q = lane; q < N * p.TH; q += 32) b[L.hist + q] = 0;
         for (int i = lane; i < NK; i += 32) {
             reinterpret_cast<uint16_t *>(b + L.cnt)[i] = 0;
             reinterpret_cast<uint32_t *>(b + L.head)[i] = kNone;
@@ -1250,13 +1116,12 @@ __global__ void k_export_stats(const RepState *rep, sim_replica_stats_t *out, in
 // ---- launch configuration ---------------------------------------------------
 typedef void (*RunKernel)(Params);
 
-template <bool SMS>
-RunKernel pick(int c) {  // c = instances per lane
+inline RunKernel pick(int c) {  // c = instances per lane
     switch (c) {
-        case 1: return k_run<1, SMS>;
-        case 2: return k_run<2, SMS>;
-        case 4: return k_run<4, SMS>;
-        default: return k_run<8, SMS>;
+        case 1: return k_run<1>;
+        case 2: return k_run<2>;
+        case 4: return k_run<4>;
+        default: return k_run<8>;
     }
 }
 
@@ -1264,12 +1129,13 @@ struct Launch {
     RunKernel fn = nullptr;
     int grid = 0;
     size_t smem = 0;
-    uint32_t slot_bytes = 0;
 };
 
 inline int lanes_c(int N) { return N <= 32 ? 1 : N <= 64 ? 2 : N <= 128 ? 4 : 8; }
 
-inline Layout make_layout(int N, int K) {
+inline int hist_stride(int T) { return (T + 3) & ~3; }
+
+inline Layout make_layout(int N, int K, int T) {
     Layout L;
     uint32_t o = 0;
     auto take = [&](uint32_t bytes, uint32_t align) {
@@ -1286,32 +1152,32 @@ inline Layout make_layout(int N, int K) {
     L.key = take(4u * N, 16);
     L.mreq = take(4u * N, 16);
     L.mcopied = take(4u * N, 16);
+    L.nf = take(4u * N, 16);
+    L.minfin = take(4u * N, 16);
     L.head = take(4u * N * K, 16);
     L.tail = take(4u * N * K, 16);
     L.h = take(4u * K, 16);
     L.wmask = take(2u * N, 16);
     L.cnt = take(2u * N * K, 16);
     L.nrun = take(N, 16);
-    L.nb = take(N, 16);
+    L.pc = take(N, 16);
+    L.phase = take(N, 16);
+    L.alo = take(N, 16);
+    L.ahi = take(N, 16);
     L.mrole = take(N, 16);
     L.mpeer = take(N, 16);
+    L.hist = take((uint32_t)N * hist_stride(T), 16);
     L.bytes = (o + 15u) & ~15u;
     return L;
 }
 
 // Chooses the kernel variant and grid for a problem; cudaSuccess or the error.
-// Odd slot stride per instance (>= Bmax), so lanes walking different instances hit different banks.
-inline int slot_stride(int Bmax) { return Bmax | 1; }
-inline uint32_t slots_per_replica(int N, int SP) { return ((uint32_t)N * (uint32_t)SP + 3u) & ~3u; }
 inline uint32_t hash_bytes_for(int N) { return lanes_c(N) > 1 ? kHashSlots * 4u : 0u; }
 
-inline cudaError_t plan_launch(int R, int N, int SP, const Layout &L, Launch &out) {
-    const int c = lanes_c(N);
-    const uint32_t slots = slots_per_replica(N, SP) * 12u;
-    const bool sms = slots <= kSmemSlotLimit;
-    out.fn = sms ? pick<true>(c) : pick<false>(c);
-    out.slot_bytes = sms ? slots : 0u;
-    out.smem = kMagicBytes + (size_t)kWarpsPerBlock * (L.bytes + out.slot_bytes + hash_bytes_for(N));
+// Chooses the kernel variant and grid for a problem; cudaSuccess or the error.
+inline cudaError_t plan_launch(int R, int N, const Layout &L, Launch &out) {
+    out.fn = pick(lanes_c(N));
+    out.smem = kMagicBytes + (size_t)kWarpsPerBlock * (L.bytes + hash_bytes_for(N));
     int dev = 0, sms_count = 0, per_sm = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms_count, cudaDevAttrMultiProcessorCount, dev);
@@ -1336,7 +1202,7 @@ inline unsigned long long magic40(unsigned d) { return ((1ull << kMagicShift) + 
 struct sim {
     sim_cluster_t cl;
     sim_policy_t pol;
-    int K = 0, ntables = 0, SP = 0;
+    int K = 0, ntables = 0;
     std::vector<int> tbl_k, tbl_h, rep_table;
     cudaStream_t stream = nullptr;
     sim_allocator_t al{};
@@ -1348,8 +1214,7 @@ struct sim {
     size_t dev_bytes = 0;
     int *d_rep_table = nullptr, *d_tbl_k = nullptr, *d_tbl_h = nullptr;
     unsigned char *d_blobs = nullptr;
-    uint32_t *d_srid = nullptr;
-    uint64_t *d_sst = nullptr;
+    uint4 *d_slots = nullptr;
     mt::RepState *d_rep = nullptr;
     sim_migration_event_t *d_log = nullptr;
     int *d_work = nullptr;  // [0] work counter, [1] validation flags, [2] unfinished count
@@ -1416,14 +1281,13 @@ void dfree(sim_t *s, void *p) {
 
 // Fills the scalar part of the kernel parameters (pointers are set by the caller).
 void fill_scalars(mt::Params &p, const sim_cluster_t &cl, const sim_policy_t &pol, int K, int cap,
-                  const mt::Layout &L, uint32_t slot_bytes, long long max_steps) {
+                  const mt::Layout &L, long long max_steps) {
     p.R = cl.num_replicas;
     p.N = cl.num_instances;
     p.M = cl.blocks_per_instance;
     p.T = cl.tokens_per_block;
     p.Bmax = cl.max_batch;
-    p.SP = mt::slot_stride(cl.max_batch);
-    p.NS = mt::slots_per_replica(cl.num_instances, p.SP);
+    p.TH = mt::hist_stride(cl.tokens_per_block);
     p.K = K;
     p.S = pol.migrate_blocks_per_iter;
     p.cap = cap;
@@ -1437,14 +1301,13 @@ void fill_scalars(mt::Params &p, const sim_cluster_t &cl, const sim_policy_t &po
     p.a = (int)pol.iter_us_per_prefill_token;
     p.b = (int)pol.iter_us_per_decode_seq;
     p.L = L;
-    p.slot_bytes = slot_bytes;
     p.hash_bytes = mt::hash_bytes_for(cl.num_instances);
 }
 
 mt::Params make_params(const sim_t *s, long long max_steps) {
     mt::Params p;
     memset(&p, 0, sizeof p);
-    fill_scalars(p, s->cl, s->pol, s->K, s->pol.event_log_capacity, s->L, s->launch.slot_bytes, max_steps);
+    fill_scalars(p, s->cl, s->pol, s->K, s->pol.event_log_capacity, s->L, max_steps);
     p.offsets = s->d_off;
     p.arrival = s->d_arrival;
     p.plen = s->d_plen;
@@ -1454,8 +1317,7 @@ mt::Params make_params(const sim_t *s, long long max_steps) {
     p.link = s->d_link;
     p.res = s->d_res;
     p.blobs = s->d_blobs;
-    p.srid = s->d_srid;
-    p.sst = s->d_sst;
+    p.slots = s->d_slots;
     p.rep = s->d_rep;
     p.log = s->d_log;
     p.work = s->d_work;
@@ -1490,8 +1352,8 @@ int validate_config(sim_t *s, const sim_cluster_t *cl, const sim_tier_table_t *t
         return fail(s, SIM_ERR_ARG, "num_instances must be in [1, %d]", SIM_MAX_INSTANCES);
     if (cl->blocks_per_instance < 1 || cl->blocks_per_instance > SIM_MAX_BLOCKS)
         return fail(s, SIM_ERR_ARG, "blocks_per_instance must be in [1, %d]", SIM_MAX_BLOCKS);
-    if (cl->tokens_per_block < 1 || cl->tokens_per_block > 65535)
-        return fail(s, SIM_ERR_ARG, "tokens_per_block must be in [1, 65535]");
+    if (cl->tokens_per_block < 1 || cl->tokens_per_block > mt::kMaxBlockTokens)
+        return fail(s, SIM_ERR_ARG, "tokens_per_block must be in [1, %d]", mt::kMaxBlockTokens);
     if (cl->max_batch < 1 || cl->max_batch > SIM_MAX_BATCH)
         return fail(s, SIM_ERR_ARG, "max_batch must be in [1, %d]", SIM_MAX_BATCH);
     if (tt->num_tables < 1 || tt->max_tiers < 1 || tt->max_tiers > SIM_MAX_TIERS)
@@ -1569,25 +1431,23 @@ int sim_create(const sim_cluster_t *cl, const sim_tier_table_t *tt, const sim_po
     s->pol = *pol;
     s->K = tt->max_tiers;
     s->ntables = tt->num_tables;
-    s->SP = mt::slot_stride(cl->max_batch);
     s->tbl_k.assign(tt->num_tiers, tt->num_tiers + tt->num_tables);
     s->tbl_h.assign(tt->headroom_blocks, tt->headroom_blocks + (size_t)tt->num_tables * tt->max_tiers);
     s->rep_table.assign(tt->replica_table, tt->replica_table + cl->num_replicas);
     s->stream = (cudaStream_t)cuda_stream;
     if (allocator) { s->al = *allocator; s->use_al = true; }
-    s->L = mt::make_layout(cl->num_instances, s->K);
+    s->L = mt::make_layout(cl->num_instances, s->K, cl->tokens_per_block);
 
-    const size_t R = (size_t)cl->num_replicas, NS = mt::slots_per_replica(cl->num_instances, s->SP);
+    const size_t R = (size_t)cl->num_replicas, NB = (size_t)cl->num_instances * cl->max_batch;
     s->d_rep_table = (int *)dalloc(s, R * 4);
     s->d_tbl_k = (int *)dalloc(s, (size_t)s->ntables * 4);
     s->d_tbl_h = (int *)dalloc(s, (size_t)s->ntables * s->K * 4);
     s->d_blobs = (unsigned char *)dalloc(s, R * s->L.bytes);
-    s->d_srid = (uint32_t *)dalloc(s, R * NS * 4);
-    s->d_sst = (uint64_t *)dalloc(s, R * NS * 8);
+    s->d_slots = (uint4 *)dalloc(s, R * NB * 16);
     s->d_rep = (mt::RepState *)dalloc(s, R * sizeof(mt::RepState));
     s->d_log = (sim_migration_event_t *)dalloc(s, R * (size_t)pol->event_log_capacity * sizeof(sim_migration_event_t));
     s->d_work = (int *)dalloc(s, 16);
-    if (!s->d_rep_table || !s->d_tbl_k || !s->d_tbl_h || !s->d_blobs || !s->d_srid || !s->d_sst || !s->d_rep ||
+    if (!s->d_rep_table || !s->d_tbl_k || !s->d_tbl_h || !s->d_blobs || !s->d_slots || !s->d_rep ||
         !s->d_log || !s->d_work) {
         const size_t held = s->dev_bytes;
         sim_destroy(s);
@@ -1602,7 +1462,7 @@ int sim_create(const sim_cluster_t *cl, const sim_tier_table_t *tt, const sim_po
     int dev = 0;
     if (e == cudaSuccess) e = cudaGetDevice(&dev);
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&s->sms, cudaDevAttrMultiProcessorCount, dev);
-    if (e == cudaSuccess) e = mt::plan_launch(cl->num_replicas, cl->num_instances, s->SP, s->L, s->launch);
+    if (e == cudaSuccess) e = mt::plan_launch(cl->num_replicas, cl->num_instances, s->L, s->launch);
     if (e != cudaSuccess) {
         cudaGetLastError();
         rc = e == cudaErrorInvalidConfiguration
@@ -1802,13 +1662,11 @@ extern "C" int sim_run_static(const sim_cluster_t *cl, const sim_tier_table_t *t
     const int cap = events ? pol->event_log_capacity : 0;
 
     // Carve the scratch array.
-    const int N = cl->num_instances, SP = mt::slot_stride(cl->max_batch), K = tt->max_tiers;
-    const mt::Layout L = mt::make_layout(N, K);
+    const int N = cl->num_instances, K = tt->max_tiers;
+    const mt::Layout L = mt::make_layout(N, K, cl->tokens_per_block);
     size_t o = 0;
     const size_t o_blobs = o; o = align256(o + (size_t)R * L.bytes);
-    const size_t NS = mt::slots_per_replica(N, SP);
-    const size_t o_srid = o; o = align256(o + (size_t)R * NS * 4);
-    const size_t o_sst = o; o = align256(o + (size_t)R * NS * 8);
+    const size_t o_slots = o; o = align256(o + (size_t)R * N * cl->max_batch * 16);
     const size_t o_rep = o; o = align256(o + (size_t)R * sizeof(mt::RepState));
     const size_t o_g = o; o = align256(o + (size_t)n * 2);
     const size_t o_link = o; o = align256(o + (size_t)n * 8);
@@ -1836,7 +1694,7 @@ extern "C" int sim_run_static(const sim_cluster_t *cl, const sim_tier_table_t *t
     cudaStream_t st = (cudaStream_t)cuda_stream;
 
     mt::Launch lc;
-    e = mt::plan_launch(R, N, SP, L, lc);
+    e = mt::plan_launch(R, N, L, lc);
     if (e != cudaSuccess) {
         cudaGetLastError();
         return e == cudaErrorInvalidConfiguration
@@ -1845,7 +1703,7 @@ extern "C" int sim_run_static(const sim_cluster_t *cl, const sim_tier_table_t *t
     }
     mt::Params p;
     memset(&p, 0, sizeof p);
-    fill_scalars(p, *cl, *pol, K, cap, L, lc.slot_bytes, 1LL << 62);
+    fill_scalars(p, *cl, *pol, K, cap, L, 1LL << 62);
     p.offsets = (const long long *)(base + o_off);
     p.arrival = arrival;
     p.plen = plen;
@@ -1855,8 +1713,7 @@ extern "C" int sim_run_static(const sim_cluster_t *cl, const sim_tier_table_t *t
     p.link = (uint2 *)(base + o_link);
     p.res = per_request;
     p.blobs = base + o_blobs;
-    p.srid = (uint32_t *)(base + o_srid);
-    p.sst = (uint64_t *)(base + o_sst);
+    p.slots = (uint4 *)(base + o_slots);
     p.rep = (mt::RepState *)(base + o_rep);
     p.log = events;
     p.work = (int *)(base + o_work);

@@ -56,7 +56,8 @@ def _valid():
 
 @pytest.mark.parametrize("field,value", [
     ("num_replicas", 0), ("num_instances", 0), ("num_instances", 257), ("blocks_per_instance", 0),
-    ("blocks_per_instance", 65536), ("tokens_per_block", 0), ("max_batch", 0), ("max_batch", 65)])
+    ("blocks_per_instance", 65536), ("tokens_per_block", 0), ("tokens_per_block", 65), ("max_batch", 0),
+    ("max_batch", 65)])
 def test_create_rejects_bad_cluster(L, field, value):
     cl, tt, pol, keep = _valid()
     setattr(cl, field, value)
@@ -67,7 +68,7 @@ def test_create_rejects_bad_cluster(L, field, value):
 
 
 @pytest.mark.parametrize("field,value", [
-    ("policy", 3), ("enable_migration", 2), ("iter_base_us", -1), ("iter_us_per_decode_seq", 1 << 25),
+    ("policy", 3), ("enable_migration", 2), ("iter_base_us", -1), ("iter_base_us", 0), ("iter_us_per_decode_seq", 1 << 25),
     ("migrate_blocks_per_iter", 0), ("theta_den", 0), ("theta_num", -1), ("event_log_capacity", -5),
     ("migrate_interval_us", 0), ("migrate_interval_us", 1 << 32)])
 def test_create_rejects_bad_policy(L, field, value):
