@@ -93,6 +93,7 @@ struct Layout {
     uint32_t head, tail;                                                 // [N*K] x 4 B
     uint32_t h;                                                          // [K] x 4 B
     uint32_t hist;                                                       // [N*TH] x 1 B
+    uint32_t mslot;                                                      // [N] x 16 B
     uint32_t bytes;
 };
 
@@ -135,6 +136,7 @@ struct Ctx {
     int *free_, *resv, *hol, *hr, *key, *mcopied, *h;
     uint16_t *wmask, *cnt;
     uint8_t *nrun, *pc, *phase, *alo, *ahi, *mrole, *mpeer, *hist;
+    uint4 *mslot;                     // record of the request a migration source is copying out
     uint4 *slots;
     uint32_t *tset;                   // event-time set (C > 1)
     const unsigned long long *magic;  // [65]: ceil(2^64 / d) for d >= 2
@@ -376,33 +378,15 @@ __device__ __forceinline__ void commit_mig(const Ctx &x, Cnt &cn, int s, int pos
     clear_mig(x, s, d);
 }
 
-// One copy stage at the end of an iteration of migration source s.
-__device__ __forceinline__ void migration_stage(const Ctx &x, Cnt &cn, int s) {
-    const int d = x.mpeer[s];
-    const uint32_t rid = x.mreq[s];
-    const uint4 *p = slot_ptr(x, s, 0);
-    int pos = -1;
-    for (int q = 0, n = x.nrun[s]; q < n; ++q)
-        if (p[q].x == rid) { pos = q; break; }
-    if (pos < 0) { cn.status = SIM_ERR_INTERNAL; return; }
-    const int blocks = sl_blocks(x, s, p[pos]);
-    const int cp = x.mcopied[s];
-    const int cc = min(x.S, blocks - cp);
-    if (x.free_[d] < cc) { abort_mig(x, cn, s); return; }
-    x.free_[d] -= cc;
-    x.resv[d] += cc;
-    x.mcopied[s] = cp + cc;
-    if (cp + cc == blocks && (int)x.nrun[d] < x.Bmax) commit_mig(x, cn, s, pos);
-}
-
-// Phase 1: the iteration of instance i ends at x.t (Sec. 2.1 token accounting):
-// fresh requests get their first token, requests whose output is complete
-// finish and free their KV, and a migration source runs one copy stage.
-__device__ __forceinline__ void inst_complete(const Ctx &x, Cnt &cn, int i) {
+// Phase 1, first part, single thread: the iteration of instance i ends at
+// x.t (Sec. 2.1 token accounting): the last formation's fresh admissions get
+// their first token.  Returns whether some running request finishes now
+// (then coop_finish must run before anything else touches instance i).
+__device__ __forceinline__ bool inst_complete_head(const Ctx &x, Cnt &cn, int i) {
     x.busy[i] = kNone;
     x.pc[i] = 1;
     uint4 *p = slot_ptr(x, i, 0);
-    for (int s = x.alo[i], e = x.ahi[i]; s < e; ++s) {  // the last formation's admissions
+    for (int s = x.alo[i], e = x.ahi[i]; s < e; ++s) {
         uint4 sl = p[s];
         if (sl.w & kFirstFlag) {
             x.res[sl.x].first_token_us = x.t;
@@ -412,30 +396,94 @@ __device__ __forceinline__ void inst_complete(const Ctx &x, Cnt &cn, int i) {
         }
     }
     x.alo[i] = x.ahi[i] = 0;
+    return x.minfin[i] == x.nf[i];
+}
+
+// Phase 1, second part, whole warp: the requests of instance i whose output
+// is complete finish at x.t and free their KV (an in-flight migration of one
+// of them is abandoned).  Lane l looks at slots l and 32 + l.
+__device__ __forceinline__ void coop_finish(const Ctx &x, Cnt &cn, int i) {
+    const int n = x.nrun[i];
     const uint32_t nf = x.nf[i];
-    if (x.minfin[i] == nf) {
-        int w = 0;
-        uint32_t m = kNone;
-        for (int s = 0, n = x.nrun[i]; s < n; ++s) {
-            const uint4 sl = p[s];
-            if (sl_fin(sl) == nf) {
-                x.res[sl.x].finish_us = x.t;
-                x.res[sl.x].final_instance = (uint16_t)i;
-                x.free_[i] += sl_blocks(x, i, sl);
-                cnt_dec(x, i, (int)sl_tier(sl));
-                x.hist[i * x.TH + sl_rho(sl)]--;
-                cn.finished++;
-                cn.events++;
-                if (x.mrole[i] == MIG_SRC && x.mreq[i] == sl.x) abort_mig(x, cn, i);
-            } else {
-                p[w++] = sl;
-                m = min(m, sl_fin(sl));
+    uint4 *p = slot_ptr(x, i, 0);
+    const int q0 = x.lane, q1 = x.lane + 32;
+    const bool v0 = q0 < n, v1 = q1 < n;
+    const uint4 a0 = v0 ? p[q0] : make_uint4(0, 0, 0, 0);
+    const uint4 a1 = v1 ? p[q1] : make_uint4(0, 0, 0, 0);
+    const bool f0 = v0 && sl_fin(a0) == nf, f1 = v1 && sl_fin(a1) == nf;
+    if (f0) { x.res[a0.x].finish_us = x.t; x.res[a0.x].final_instance = (uint16_t)i; }
+    if (f1) { x.res[a1.x].finish_us = x.t; x.res[a1.x].final_instance = (uint16_t)i; }
+    const int freed = __reduce_add_sync(kFull, (f0 ? sl_blocks(x, i, a0) : 0) + (f1 ? sl_blocks(x, i, a1) : 0));
+    const uint32_t m0 = __ballot_sync(kFull, f0), m1 = __ballot_sync(kFull, f1);
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+        uint32_t lanes = j ? m1 : m0;
+        while (lanes) {
+            const int l = __ffs(lanes) - 1;
+            lanes &= lanes - 1;
+            const uint32_t rid = __shfl_sync(kFull, j ? a1.x : a0.x, l);
+            const uint32_t w = __shfl_sync(kFull, j ? a1.w : a0.w, l);
+            if (x.lane == 0) {
+                cnt_dec(x, i, (int)(w & 0xFFu));
+                x.hist[i * x.TH + (w >> 16)]--;
+                if (x.mrole[i] == MIG_SRC && x.mreq[i] == rid) abort_mig(x, cn, i);
             }
         }
-        x.nrun[i] = (uint8_t)w;
-        x.minfin[i] = m;
     }
-    if (x.mrole[i] == MIG_SRC) migration_stage(x, cn, i);
+    const bool k0 = v0 && !f0, k1 = v1 && !f1;
+    const uint32_t e0 = __ballot_sync(kFull, k0), e1 = __ballot_sync(kFull, k1);
+    const uint32_t below = (1u << x.lane) - 1u;
+    const int p0 = __popc(e0 & below), p1 = __popc(e0) + __popc(e1 & below);
+    const uint32_t fm = __reduce_min_sync(kFull, min(k0 ? sl_fin(a0) : kNone, k1 ? sl_fin(a1) : kNone));
+    __syncwarp();
+    if (k0) p[p0] = a0;
+    if (k1) p[p1] = a1;
+    if (x.lane == 0) {
+        const uint32_t nfin = __popc(m0) + __popc(m1);
+        x.free_[i] += freed;
+        x.nrun[i] = (uint8_t)(__popc(e0) + __popc(e1));
+        x.minfin[i] = fm;
+        cn.finished += nfin;
+        cn.events += nfin;
+    }
+    __syncwarp();
+}
+
+// One copy stage at the end of an iteration of migration source s, whole
+// warp: up to S of the request's blocks are reserved on the destination
+// (abandoning the migration if they do not fit), and the request commits
+// there once all of them are copied (Sec. 3.5, Fig. 4).
+__device__ __forceinline__ void coop_stage(const Ctx &x, Cnt &cn, int s) {
+    int commit = 0;
+    if (x.lane == 0) {
+        const int d = x.mpeer[s];
+        const int blocks = sl_blocks(x, s, x.mslot[s]);
+        const int cp = x.mcopied[s];
+        const int cc = min(x.S, blocks - cp);
+        if (x.free_[d] < cc) {
+            abort_mig(x, cn, s);
+        } else {
+            x.free_[d] -= cc;
+            x.resv[d] += cc;
+            x.mcopied[s] = cp + cc;
+            commit = (cp + cc == blocks) && ((int)x.nrun[d] < x.Bmax);
+        }
+    }
+    commit = __shfl_sync(kFull, commit, 0);
+    __syncwarp();
+    if (commit) {
+        const uint32_t rid = x.mreq[s];
+        const int n = x.nrun[s];
+        const uint4 *p = slot_ptr(x, s, 0);
+        const uint32_t h0 = __ballot_sync(kFull, x.lane < n && p[x.lane].x == rid);
+        const uint32_t h1 = __ballot_sync(kFull, x.lane + 32 < n && p[x.lane + 32].x == rid);
+        const int pos = h0 ? __ffs(h0) - 1 : (h1 ? 32 + __ffs(h1) - 1 : -1);
+        if (x.lane == 0) {
+            if (pos < 0) cn.status = SIM_ERR_INTERNAL;
+            else commit_mig(x, cn, s, pos);
+        }
+        __syncwarp();
+    }
 }
 
 // Recompute-style preemption of running request `sl` (holding `blocks` KV
@@ -655,9 +703,12 @@ __device__ __forceinline__ void migration_tick(const Ctx &x, Cnt &cn, int theta_
         const long long ns = fnum(x, s), ds = max((int)x.nrun[s], 1);
         const long long nd = fnum(x, d), dd = max((int)x.nrun[d], 1);
         if ((long long)theta_den * (nd * ds - ns * dd) < (long long)theta_num * dd * ds) break;
+        const bool has_wait = x.wmask[s] != 0;
+        const int n_s = x.nrun[s];
+        __syncwarp();
         int moved = 0;
-        if (x.lane == 0) {
-            if (x.wmask[s] != 0) {
+        if (has_wait) {
+            if (x.lane == 0) {
                 // queued candidate: newest request of the lowest-priority bucket, no KV to copy
                 const int k = 31 - __clz((unsigned)x.wmask[s]);
                 const uint32_t r = pop_back(x, s, k, cn.status);
@@ -673,33 +724,44 @@ __device__ __forceinline__ void migration_tick(const Ctx &x, Cnt &cn, int theta_
                     cn.events++;
                     log_ev(x, cn, SIM_EV_QUEUED, r, s, d, 0);
                 }
-                moved = 1;
-            } else if (x.nrun[s] > 0) {
-                // running candidate: lowest priority, then fewest blocks, then newest
-                const uint4 *p = slot_ptr(x, s, 0);
-                int best = -1, bb = 0;
-                uint32_t bt = 0, br = 0;
-                for (int q = 0, n = x.nrun[s]; q < n; ++q) {
-                    const uint32_t tq = sl_tier(p[q]), rq = p[q].x;
-                    const int bq = sl_blocks(x, s, p[q]);
-                    if (best < 0 || tq > bt || (tq == bt && (bq < bb || (bq == bb && rq > br)))) {
-                        best = q; bt = tq; bb = bq; br = rq;
-                    }
-                }
-                if (x.free_[d] >= bb) {
+            }
+            moved = 1;
+        } else if (n_s > 0) {
+            // running candidate: lowest priority, then fewest blocks, then newest
+            const uint4 *p = slot_ptr(x, s, 0);
+            const bool v0 = x.lane < n_s, v1 = x.lane + 32 < n_s;
+            const uint4 a0 = v0 ? p[x.lane] : make_uint4(0, 0, 0, 0);
+            const uint4 a1 = v1 ? p[x.lane + 32] : make_uint4(0, 0, 0, 0);
+            const int k0 = v0 ? (int)((sl_tier(a0) << 16) | (0xFFFFu - (uint32_t)sl_blocks(x, s, a0))) : -1;
+            const int k1 = v1 ? (int)((sl_tier(a1) << 16) | (0xFFFFu - (uint32_t)sl_blocks(x, s, a1))) : -1;
+            const int km = __reduce_max_sync(kFull, max(k0, k1));
+            const uint32_t c0 = (v0 && k0 == km) ? a0.x : 0u, c1 = (v1 && k1 == km) ? a1.x : 0u;
+            const uint32_t rid = __reduce_max_sync(kFull, max(c0, c1));
+            const int blocks = (int)(0xFFFFu - ((uint32_t)km & 0xFFFFu));
+            const uint32_t o0 = __ballot_sync(kFull, v0 && a0.x == rid);
+            const uint32_t o1 = __ballot_sync(kFull, v1 && a1.x == rid);
+            const int ol = o0 ? __ffs(o0) - 1 : __ffs(o1) - 1;
+            const bool hi = o0 == 0;
+            uint4 rec;
+            rec.x = __shfl_sync(kFull, hi ? a1.x : a0.x, ol);
+            rec.y = __shfl_sync(kFull, hi ? a1.y : a0.y, ol);
+            rec.z = __shfl_sync(kFull, hi ? a1.z : a0.z, ol);
+            rec.w = __shfl_sync(kFull, hi ? a1.w : a0.w, ol);
+            if (x.free_[d] >= blocks) {
+                if (x.lane == 0) {
                     x.mrole[s] = MIG_SRC;
                     x.mpeer[s] = (uint8_t)d;
-                    x.mreq[s] = br;
+                    x.mreq[s] = rid;
                     x.mcopied[s] = 0;
+                    x.mslot[s] = rec;
                     x.mrole[d] = MIG_DST;
                     x.mpeer[d] = (uint8_t)s;
                     cn.starts++;
-                    log_ev(x, cn, SIM_EV_START, br, s, d, bb);
-                    moved = 1;
+                    log_ev(x, cn, SIM_EV_START, rid, s, d, blocks);
                 }
+                moved = 1;
             }
         }
-        moved = __shfl_sync(kFull, moved, 0);
         if (x.lane == s / C) el &= ~(1u << (s % C));
         if (moved && x.lane == d / C) el &= ~(1u << (d % C));
         __syncwarp();
@@ -747,10 +809,11 @@ __device__ __forceinline__ void bind_blob(Ctx &x, const Layout &L, unsigned char
     x.tail = reinterpret_cast<uint32_t *>(blob + L.tail);
     x.h = reinterpret_cast<int *>(blob + L.h);
     x.hist = blob + L.hist;
+    x.mslot = reinterpret_cast<uint4 *>(blob + L.mslot);
 }
 
 // Phase 1 at x.t for the instances in `mask` (bit j = instance lane*C + j)
-// whose iteration ends now, ascending index, on lane 0.  Collective.
+// whose iteration ends now, ascending index.  Collective.
 template <int C>
 __device__ __forceinline__ void complete_all(const Ctx &x, Cnt &cn, uint32_t mask) {
     uint32_t hits = 0;
@@ -761,11 +824,17 @@ __device__ __forceinline__ void complete_all(const Ctx &x, Cnt &cn, uint32_t mas
     while (lanes) {
         const int l = __ffs(lanes) - 1;
         lanes &= lanes - 1;
-        const uint32_t h = C == 1 ? 1u : __shfl_sync(kFull, hits, l);
-        if (x.lane == 0)
-            for (uint32_t hh = h; hh; hh &= hh - 1) inst_complete(x, cn, l * C + __ffs(hh) - 1);
+        uint32_t h = C == 1 ? 1u : __shfl_sync(kFull, hits, l);
+        while (h) {
+            const int i = l * C + __ffs(h) - 1;
+            h &= h - 1;
+            int fp = 0;
+            if (x.lane == 0) fp = inst_complete_head(x, cn, i);
+            if (__shfl_sync(kFull, fp, 0)) coop_finish(x, cn, i);
+            __syncwarp();
+            if (x.mrole[i] == MIG_SRC) coop_stage(x, cn, i);
+        }
     }
-    __syncwarp();
 }
 
 // Phase 4 at x.t for the idle instances in `mask` that have work, ascending
@@ -858,7 +927,6 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
         cn.member_iterations = l0 ? rs.member_iterations : 0ull;
         cn.events = l0 ? rs.events : 0ull;
         cn.status = SIM_REPLICA_RUNNING;
-        uint32_t wfin = 0;  // requests this lane finished in the current window
         uint32_t cursor = rs.cursor;
         uint32_t next_tick = rs.next_tick;
         ArrBuf ab;
@@ -897,7 +965,7 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
                 }
                 uint32_t fresh = 0;  // distinct event times this lane contributes (C > 1)
                 uint32_t tlast = 0;  // latest event time processed in the window
-                const uint32_t fin0 = cn.finished;
+                uint32_t pend = 0;   // instances whose finishing requests the warp handles next
 #pragma unroll
                 for (int j = 0; j < C; ++j) {
                     if (!((solo >> j) & 1u)) continue;
@@ -905,12 +973,27 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
                     x.t = bz[j];
                     tlast = max(tlast, bz[j]);
                     if (C > 1) fresh += tset_insert(x, bz[j]);
-                    inst_complete(x, cn, i);
-                    inst_form(x, cn, i, p.base, p.a, p.b);
+                    if (inst_complete_head(x, cn, i)) pend |= 1u << j;
+                    else inst_form(x, cn, i, p.base, p.a, p.b);
                 }
-                wfin = cn.finished - fin0;
-                cn.finished = fin0;
                 __syncwarp();
+                {
+                    uint32_t pl = __ballot_sync(kFull, pend != 0);
+                    while (pl) {
+                        const int l = __ffs(pl) - 1;
+                        pl &= pl - 1;
+                        uint32_t h = C == 1 ? 1u : __shfl_sync(kFull, pend, l);
+                        while (h) {
+                            const int j = __ffs(h) - 1;
+                            h &= h - 1;
+                            const int i = l * C + j;
+                            x.t = __shfl_sync(kFull, bz[j], l);
+                            coop_finish(x, cn, i);
+                            if (lane == 0) inst_form(x, cn, i, p.base, p.a, p.b);
+                            __syncwarp();
+                        }
+                    }
+                }
                 uint32_t ucount, u = kNone;
                 if (C == 1) {
                     u = solo ? bz[0] : kNone;
@@ -936,11 +1019,8 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
                         if (tc >= t1) break;
                         x.t = tc;
                         tlast = max(tlast, tc);
-                        const uint32_t f1 = cn.finished;
                         complete_all<C>(x, cn, cm);
                         form_all<C>(x, cn, cm, p);
-                        wfin += __shfl_sync(kFull, cn.finished - f1, 0) * (lane == 0 ? 1u : 0u);
-                        cn.finished = __shfl_sync(kFull, f1, 0);
                         if (C == 1) {
                             ucount += __any_sync(kFull, u == tc) ? 0u : 1u;
                         } else {
@@ -954,7 +1034,7 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
                 }
                 cn.steps += ucount;
                 x.t = __reduce_max_sync(kFull, tlast);
-                cn.finished += __reduce_add_sync(kFull, wfin);
+                cn.finished = __shfl_sync(kFull, cn.finished, 0);  // finishes are all counted on lane 0
                 const int ws = __reduce_min_sync(kFull, cn.status);
                 cn.status = ws;
                 if (cn.status < 0) break;
@@ -1167,6 +1247,7 @@ inline Layout make_layout(int N, int K, int T) {
     L.mrole = take(N, 16);
     L.mpeer = take(N, 16);
     L.hist = take((uint32_t)N * hist_stride(T), 16);
+    L.mslot = take(16u * N, 16);
     L.bytes = (o + 15u) & ~15u;
     return L;
 }
