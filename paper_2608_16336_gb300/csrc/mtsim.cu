@@ -74,7 +74,7 @@ enum : int { MIG_NONE = 0, MIG_SRC = 1, MIG_DST = 2 };
 //   x = request id (index in the replica's trace)
 //   y = phi: number of the instance's first formation that includes it
 //   z = c | left << 16: its context length P + g and its remaining output O - g at formation phi
-//   w = tier | flags << 8 | rho << 16, rho = (c - phi) mod T
+//   w = tier | rho << 16, rho = (c - phi) mod T
 // With nf formations done and pc = 1 after the iteration that followed the
 // last one (0 before), the request has advanced adv = nf - phi + pc tokens
 // (0 if phi > nf) and holds ceil((c + nf - phi) / T) KV blocks: every
@@ -83,14 +83,20 @@ enum : int { MIG_NONE = 0, MIG_SRC = 1, MIG_DST = 2 };
 // requests that need a new block at the next formation is the count of
 // running requests with rho == -nf (mod T), and a request finishes at the
 // iteration that follows formation phi + left - 1.
-constexpr uint32_t kFirstFlag = 1u << 8;  // fresh request: its first token is due at the next iteration end
+constexpr uint32_t kFreshFlag = 1u << 8;  // set between admission and the end of formation: no token yet
+
+// A waiting request's queue node (16 bytes, indexed by request) carries what
+// admitting it needs: x = next, y = info of next, z = prev, w = own info, with
+// info = context (P + g) | remaining output (O - g) << 16.  The info of each
+// bucket's head is also kept in shared memory, so admission and the HoL demand
+// need no dependent HBM reads.
 
 struct Layout {
     uint32_t busy, free_, resv, hol, hr, key, mreq, mcopied, nf, minfin;  // [N] x 4 B
     uint32_t wmask;                                                      // [N] x 2 B
-    uint32_t nrun, pc, phase, alo, ahi, mrole, mpeer;                     // [N] x 1 B
+    uint32_t nrun, pc, phase, mrole, mpeer;                               // [N] x 1 B
     uint32_t cnt;                                                        // [N*K] x 2 B
-    uint32_t head, tail;                                                 // [N*K] x 4 B
+    uint32_t head, tail, hinfo;                                          // [N*K] x 4 B
     uint32_t h;                                                          // [K] x 4 B
     uint32_t hist;                                                       // [N*TH] x 1 B
     uint32_t mslot;                                                      // [N] x 16 B
@@ -118,8 +124,7 @@ struct Params {
     const uint32_t *arrival;
     const uint16_t *plen, *olen;
     const uint8_t *tier;
-    uint16_t *g;
-    uint2 *link;  // .x = next, .y = prev
+    uint4 *node;                  // queue node per request: next, info of next, prev, own info
     sim_request_result_t *res;
     unsigned char *blobs;
     uint4 *slots;                 // [R][N][Bmax]
@@ -132,10 +137,10 @@ struct Params {
 // memory, request state and slot records in HBM; scalars are warp-uniform
 // except t while lanes advance their own instances.
 struct Ctx {
-    uint32_t *busy, *mreq, *head, *tail, *nf, *minfin;
+    uint32_t *busy, *mreq, *head, *tail, *hinfo, *nf, *minfin;
     int *free_, *resv, *hol, *hr, *key, *mcopied, *h;
     uint16_t *wmask, *cnt;
-    uint8_t *nrun, *pc, *phase, *alo, *ahi, *mrole, *mpeer, *hist;
+    uint8_t *nrun, *pc, *phase, *mrole, *mpeer, *hist;
     uint4 *mslot;                     // record of the request a migration source is copying out
     uint4 *slots;
     uint32_t *tset;                   // event-time set (C > 1)
@@ -143,8 +148,7 @@ struct Ctx {
     const uint32_t *arrival;
     const uint16_t *plen, *olen;
     const uint8_t *tier;
-    uint16_t *g;
-    uint2 *link;
+    uint4 *node;
     sim_request_result_t *res;
     sim_migration_event_t *log;
     unsigned long long magT;
@@ -232,48 +236,51 @@ __device__ __forceinline__ void cnt_inc(const Ctx &x, int i, int k) {
 __device__ __forceinline__ void cnt_dec(const Ctx &x, int i, int k) {
     if (--x.cnt[i * x.K + k] == 0) x.hr[i] -= x.h[k];
 }
-__device__ __forceinline__ void push_back(const Ctx &x, int i, int k, uint32_t r) {
+__device__ __forceinline__ void push_back(const Ctx &x, int i, int k, uint32_t r, uint32_t info) {
     const int b = i * x.K + k;
     const uint32_t tl = x.tail[b];
-    x.link[r] = make_uint2(kNone, tl);
-    if (tl != kNone) x.link[tl].x = r; else x.head[b] = r;
+    x.node[r] = make_uint4(kNone, 0u, tl, info);
+    if (tl != kNone) *reinterpret_cast<uint2 *>(&x.node[tl]) = make_uint2(r, info);
+    else { x.head[b] = r; x.hinfo[b] = info; }
     x.tail[b] = r;
     x.wmask[i] |= (uint16_t)(1u << k);
 }
-__device__ __forceinline__ void push_front(const Ctx &x, int i, int k, uint32_t r) {
+__device__ __forceinline__ void push_front(const Ctx &x, int i, int k, uint32_t r, uint32_t info) {
     const int b = i * x.K + k;
     const uint32_t hd = x.head[b];
-    x.link[r] = make_uint2(hd, kNone);
-    if (hd != kNone) x.link[hd].y = r; else x.tail[b] = r;
+    x.node[r] = make_uint4(hd, hd != kNone ? x.hinfo[b] : 0u, kNone, info);
+    if (hd != kNone) x.node[hd].z = r; else x.tail[b] = r;
     x.head[b] = r;
+    x.hinfo[b] = info;
     x.wmask[i] |= (uint16_t)(1u << k);
 }
+// Removes the head of bucket (i, k); its info is hinfo before the call.
 __device__ __forceinline__ uint32_t pop_front(const Ctx &x, int i, int k, int &status) {
     const int b = i * x.K + k;
     const uint32_t r = x.head[b];
     if (r >= x.Q) { status = SIM_ERR_INTERNAL; return kNone; }
-    const uint32_t nx = x.link[r].x;
-    x.head[b] = nx;
-    if (nx != kNone) x.link[nx].y = kNone;
+    const uint4 nd = x.node[r];
+    x.head[b] = nd.x;
+    if (nd.x != kNone) { x.node[nd.x].z = kNone; x.hinfo[b] = nd.y; }
     else { x.tail[b] = kNone; x.wmask[i] &= (uint16_t)~(1u << k); }
     return r;
 }
-__device__ __forceinline__ uint32_t pop_back(const Ctx &x, int i, int k, int &status) {
+// Removes the tail of bucket (i, k) and returns its info in `info`.
+__device__ __forceinline__ uint32_t pop_back(const Ctx &x, int i, int k, uint32_t &info, int &status) {
     const int b = i * x.K + k;
     const uint32_t r = x.tail[b];
     if (r >= x.Q) { status = SIM_ERR_INTERNAL; return kNone; }
-    const uint32_t pv = x.link[r].y;
-    x.tail[b] = pv;
-    if (pv != kNone) x.link[pv].x = kNone;
+    const uint4 nd = x.node[r];
+    info = nd.w;
+    x.tail[b] = nd.z;
+    if (nd.z != kNone) *reinterpret_cast<uint2 *>(&x.node[nd.z]) = make_uint2(kNone, 0u);
     else { x.head[b] = kNone; x.wmask[i] &= (uint16_t)~(1u << k); }
     return r;
 }
 // HoL demand: KV blocks the head of the highest-priority non-empty bucket needs.
 __device__ __forceinline__ void refresh_hol(const Ctx &x, int i) {
     const uint32_t wm = x.wmask[i];
-    if (!wm) { x.hol[i] = 0; return; }
-    const uint32_t r = x.head[i * x.K + (__ffs(wm) - 1)];
-    x.hol[i] = blocks_for(x, (uint32_t)x.plen[r] + x.g[r]);
+    x.hol[i] = wm ? blocks_for(x, x.hinfo[i * x.K + (__ffs(wm) - 1)] & 0xFFFFu) : 0;
 }
 __device__ __forceinline__ void log_ev(const Ctx &x, Cnt &cn, int kind, uint32_t r, int s, int d, int blocks) {
     const uint32_t k = cn.log_events++;
@@ -327,12 +334,12 @@ __device__ __forceinline__ uint4 *slot_ptr(const Ctx &x, int i, int s) { return 
 // A request joins instance i's running list at position n with context c and
 // remaining output left; its first formation there will be number nf + 1.
 __device__ __forceinline__ void slot_join(const Ctx &x, int i, int n, uint32_t r, uint32_t c, uint32_t left,
-                                          uint32_t tier, bool fresh) {
+                                          uint32_t tier) {
     const uint32_t phi = x.nf[i] + 1u;
     const uint32_t pm = x.phase[i] + 1u == (uint32_t)x.T ? 0u : x.phase[i] + 1u;  // phi mod T
     const uint32_t cm = mod_t(x, c);
     const uint32_t rho = cm >= pm ? cm - pm : cm + (uint32_t)x.T - pm;
-    *slot_ptr(x, i, n) = make_uint4(r, phi, c | (left << 16), tier | (fresh ? kFirstFlag : 0u) | (rho << 16));
+    *slot_ptr(x, i, n) = make_uint4(r, phi, c | (left << 16), tier | (rho << 16));
     x.hist[i * x.TH + rho]++;
     x.minfin[i] = min(x.minfin[i], phi + left - 1u);
 }
@@ -369,7 +376,7 @@ __device__ __forceinline__ void commit_mig(const Ctx &x, Cnt &cn, int s, int pos
     cnt_dec(x, s, (int)tr);
     cnt_inc(x, d, (int)tr);
     const int nd = x.nrun[d];
-    slot_join(x, d, nd, sl.x, sl_c(sl) + adv, sl_left(sl) - adv, tr, false);
+    slot_join(x, d, nd, sl.x, sl_c(sl) + adv, sl_left(sl) - adv, tr);
     x.nrun[d] = (uint8_t)(nd + 1);
     bump_mig(x, sl.x);
     cn.migrations++;
@@ -379,23 +386,12 @@ __device__ __forceinline__ void commit_mig(const Ctx &x, Cnt &cn, int s, int pos
 }
 
 // Phase 1, first part, single thread: the iteration of instance i ends at
-// x.t (Sec. 2.1 token accounting): the last formation's fresh admissions get
-// their first token.  Returns whether some running request finishes now
-// (then coop_finish must run before anything else touches instance i).
-__device__ __forceinline__ bool inst_complete_head(const Ctx &x, Cnt &cn, int i) {
+// x.t (Sec. 2.1 token accounting; first tokens were recorded when the
+// prefill iteration was scheduled).  Returns whether some running request
+// finishes now (then coop_finish must run before anything else touches i).
+__device__ __forceinline__ bool inst_complete_head(const Ctx &x, int i) {
     x.busy[i] = kNone;
     x.pc[i] = 1;
-    uint4 *p = slot_ptr(x, i, 0);
-    for (int s = x.alo[i], e = x.ahi[i]; s < e; ++s) {
-        uint4 sl = p[s];
-        if (sl.w & kFirstFlag) {
-            x.res[sl.x].first_token_us = x.t;
-            sl.w &= ~kFirstFlag;
-            p[s] = sl;
-            cn.events++;
-        }
-    }
-    x.alo[i] = x.ahi[i] = 0;
     return x.minfin[i] == x.nf[i];
 }
 
@@ -494,9 +490,8 @@ __device__ __forceinline__ void preempt_book(const Ctx &x, Cnt &cn, int i, const
     const int tr = (int)sl_tier(sl);
     const uint32_t adv = sl_adv(x, i, sl);
     x.free_[i] += blocks;
-    x.g[r] = (uint16_t)(x.olen[r] - (sl_left(sl) - adv));
     const uint32_t old = x.wmask[i];
-    push_front(x, i, tr, r);
+    push_front(x, i, tr, r, (sl_c(sl) + adv) | ((sl_left(sl) - adv) << 16));
     if ((old & ((1u << tr) - 1u)) == 0) x.hol[i] = blocks_for(x, sl_c(sl) + adv);  // now head of line
     x.hist[i * x.TH + sl_rho(sl)]--;
     bump_pre(x, r);
@@ -561,23 +556,30 @@ __device__ __forceinline__ void inst_form(const Ctx &x, Cnt &cn, int i, int base
     const int n_decode = n;
     int fr = x.free_[i];
     int prefill = 0;
-    x.alo[i] = (uint8_t)n;
+    int nfresh = 0;  // admitted requests without a token yet: their first token ends this iteration
     while (n < x.Bmax) {
         const uint32_t wm = x.wmask[i];
         if (!wm) break;
         const int need = x.hol[i];
         if (need > fr) break;
         const int k = __ffs(wm) - 1;
+        const uint32_t info = x.hinfo[i * x.K + k];
+        const uint32_t h = x.head[i * x.K + k];
+        // issued before the node read so that the two loads overlap
+        const uint32_t ft = x.res[min(h, x.Q - 1u)].first_token_us;
         const uint32_t r = pop_front(x, i, k, cn.status);
         if (r == kNone) break;
-        const uint32_t P = x.plen[r], O = x.olen[r], gg = x.g[r];
-        slot_join(x, i, n, r, P + gg, O - gg, (uint32_t)k, gg == 0);
+        const uint32_t c = info & 0xFFFFu;
+        slot_join(x, i, n, r, c, info >> 16, (uint32_t)k);
+        if (ft == kNone) {
+            slot_ptr(x, i, n)->w |= kFreshFlag;
+            ++nfresh;
+        }
         ++n;
         fr -= need;
-        prefill += (int)(P + gg);
+        prefill += (int)c;
         refresh_hol(x, i);
     }
-    x.ahi[i] = (uint8_t)n;
     x.nrun[i] = (uint8_t)n;
     x.free_[i] = fr;
     // (iii) the iteration starts
@@ -588,6 +590,17 @@ __device__ __forceinline__ void inst_form(const Ctx &x, Cnt &cn, int i, int base
             return;
         }
         x.busy[i] = (uint32_t)end;
+        if (nfresh) {
+            uint4 *sp = slot_ptr(x, i, 0);
+            for (int q = n_decode; q < n; ++q) {
+                const uint4 sl = sp[q];
+                if (sl.w & kFreshFlag) {
+                    x.res[sl.x].first_token_us = (uint32_t)end;
+                    sp[q].w = sl.w & ~kFreshFlag;
+                }
+            }
+            cn.events += (uint64_t)nfresh;
+        }
         x.nf[i] += 1u;
         x.phase[i] = x.phase[i] + 1u == (uint32_t)x.T ? (uint8_t)0 : (uint8_t)(x.phase[i] + 1u);
         x.pc[i] = 0;
@@ -599,11 +612,12 @@ __device__ __forceinline__ void inst_form(const Ctx &x, Cnt &cn, int i, int base
 // ---- cooperative steps ----------------------------------------------------------
 // Dispatch one arriving request r of tier k with prompt length P (Sec. 3.4).
 template <int C>
-__device__ __forceinline__ void dispatch_one(const Ctx &x, Cnt &cn, uint32_t r, int k, uint32_t P, uint32_t all) {
+__device__ __forceinline__ void dispatch_one(const Ctx &x, Cnt &cn, uint32_t r, int k, uint32_t P, uint32_t O,
+                                             uint32_t all) {
     const int best = arg_ext<C>(x, all, true, -1);
     if (x.lane == 0) {
         const uint32_t old = x.wmask[best];
-        push_back(x, best, k, r);
+        push_back(x, best, k, r, P | (O << 16));
         cnt_inc(x, best, k);
         if ((old & ((2u << k) - 1u)) == 0) x.hol[best] = blocks_for(x, P);  // becomes head of line
         x.res[r].dispatch_instance = (uint16_t)best;
@@ -615,7 +629,7 @@ __device__ __forceinline__ void dispatch_one(const Ctx &x, Cnt &cn, uint32_t r, 
 
 // The next 32 trace records, one per lane: index pb + lane.
 struct ArrBuf {
-    uint32_t pb, time, tier, P;
+    uint32_t pb, time, tier, P, O;
 };
 
 __device__ __forceinline__ void arr_refill(const Ctx &x, ArrBuf &ab, uint32_t cursor) {
@@ -625,6 +639,7 @@ __device__ __forceinline__ void arr_refill(const Ctx &x, ArrBuf &ab, uint32_t cu
     ab.time = in ? x.arrival[idx] : kNone;
     ab.tier = in ? (uint32_t)x.tier[idx] : 0u;
     ab.P = in ? (uint32_t)x.plen[idx] : 0u;
+    ab.O = in ? (uint32_t)x.olen[idx] : 0u;
 }
 
 // Phase 2: arrivals at t, tier 0 first, FCFS (trace order) within a tier.
@@ -650,7 +665,8 @@ __device__ __forceinline__ void dispatch_phase(const Ctx &x, Cnt &cn, uint32_t &
             while (bits) {
                 const int l = __ffs(bits) - 1;
                 bits &= bits - 1;
-                dispatch_one<C>(x, cn, ab.pb + (uint32_t)l, k, __shfl_sync(kFull, ab.P, l), all);
+                dispatch_one<C>(x, cn, ab.pb + (uint32_t)l, k, __shfl_sync(kFull, ab.P, l),
+                                __shfl_sync(kFull, ab.O, l), all);
             }
         }
         cursor += (uint32_t)__popc(eq);
@@ -671,11 +687,13 @@ __device__ __forceinline__ void dispatch_phase(const Ctx &x, Cnt &cn, uint32_t &
                 const bool mine = base + (uint32_t)x.lane < m;
                 const uint32_t tr = mine ? x.tier[j2] : 0u;
                 const uint32_t P = mine ? x.plen[j2] : 0u;
+                const uint32_t O = mine ? x.olen[j2] : 0u;
                 uint32_t bits = __ballot_sync(kFull, mine && tr == (uint32_t)k);
                 while (bits) {
                     const int l = __ffs(bits) - 1;
                     bits &= bits - 1;
-                    dispatch_one<C>(x, cn, cursor + base + (uint32_t)l, k, __shfl_sync(kFull, P, l), all);
+                    dispatch_one<C>(x, cn, cursor + base + (uint32_t)l, k, __shfl_sync(kFull, P, l),
+                                    __shfl_sync(kFull, O, l), all);
                 }
             }
         }
@@ -711,14 +729,15 @@ __device__ __forceinline__ void migration_tick(const Ctx &x, Cnt &cn, int theta_
             if (x.lane == 0) {
                 // queued candidate: newest request of the lowest-priority bucket, no KV to copy
                 const int k = 31 - __clz((unsigned)x.wmask[s]);
-                const uint32_t r = pop_back(x, s, k, cn.status);
+                uint32_t info = 0;
+                const uint32_t r = pop_back(x, s, k, info, cn.status);
                 if (r != kNone) {
                     refresh_hol(x, s);
                     cnt_dec(x, s, k);
                     const uint32_t old = x.wmask[d];
-                    push_back(x, d, k, r);
+                    push_back(x, d, k, r, info);
                     cnt_inc(x, d, k);
-                    if ((old & ((2u << k) - 1u)) == 0) x.hol[d] = blocks_for(x, (uint32_t)x.plen[r] + x.g[r]);
+                    if ((old & ((2u << k) - 1u)) == 0) x.hol[d] = blocks_for(x, info & 0xFFFFu);
                     bump_mig(x, r);
                     cn.migrations++;
                     cn.events++;
@@ -800,13 +819,12 @@ __device__ __forceinline__ void bind_blob(Ctx &x, const Layout &L, unsigned char
     x.nrun = blob + L.nrun;
     x.pc = blob + L.pc;
     x.phase = blob + L.phase;
-    x.alo = blob + L.alo;
-    x.ahi = blob + L.ahi;
     x.mrole = blob + L.mrole;
     x.mpeer = blob + L.mpeer;
     x.cnt = reinterpret_cast<uint16_t *>(blob + L.cnt);
     x.head = reinterpret_cast<uint32_t *>(blob + L.head);
     x.tail = reinterpret_cast<uint32_t *>(blob + L.tail);
+    x.hinfo = reinterpret_cast<uint32_t *>(blob + L.hinfo);
     x.h = reinterpret_cast<int *>(blob + L.h);
     x.hist = blob + L.hist;
     x.mslot = reinterpret_cast<uint4 *>(blob + L.mslot);
@@ -829,7 +847,7 @@ __device__ __forceinline__ void complete_all(const Ctx &x, Cnt &cn, uint32_t mas
             const int i = l * C + __ffs(h) - 1;
             h &= h - 1;
             int fp = 0;
-            if (x.lane == 0) fp = inst_complete_head(x, cn, i);
+            if (x.lane == 0) fp = inst_complete_head(x, i);
             if (__shfl_sync(kFull, fp, 0)) coop_finish(x, cn, i);
             __syncwarp();
             if (x.mrole[i] == MIG_SRC) coop_stage(x, cn, i);
@@ -868,7 +886,7 @@ __device__ __forceinline__ void form_all(const Ctx &x, Cnt &cn, uint32_t mask, c
 // instances (an O(1) iteration end + batch formation); instances in a
 // migration, and every step at a global event, are advanced by lane 0 in the
 // oracle's order.
-template <int C>
+template <int C, bool SMS>
 __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
     extern __shared__ __align__(16) unsigned char smem[];
     unsigned long long *magic = reinterpret_cast<unsigned long long *>(smem);
@@ -876,9 +894,11 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
         magic[d] = d < 2 ? 0ull : ~0ull / (unsigned long long)d + 1ull;
     __syncthreads();
     const int lane = threadIdx.x & 31;
-    const uint32_t per_warp = p.L.bytes + p.hash_bytes;
+    const uint32_t slot_bytes = SMS ? (uint32_t)p.N * (uint32_t)p.Bmax * 16u : 0u;
+    const uint32_t per_warp = p.L.bytes + slot_bytes + p.hash_bytes;
     unsigned char *blob = smem + kMagicBytes + (size_t)(threadIdx.x >> 5) * per_warp;
-    uint32_t *tset = reinterpret_cast<uint32_t *>(blob + p.L.bytes);
+    uint4 *sslots = reinterpret_cast<uint4 *>(blob + p.L.bytes);
+    uint32_t *tset = reinterpret_cast<uint32_t *>(blob + p.L.bytes + slot_bytes);
     for (;;) {
         int r = 0;
         if (lane == 0) r = atomicAdd(p.work, 1);
@@ -890,7 +910,14 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
         copy16(blob, gblob, p.L.bytes, lane);
         Ctx x;
         bind_blob(x, p.L, blob);
-        x.slots = p.slots + (size_t)r * p.N * p.Bmax;
+        uint4 *g_slots = p.slots + (size_t)r * p.N * p.Bmax;
+        if (SMS) {
+            copy16(reinterpret_cast<unsigned char *>(sslots), reinterpret_cast<const unsigned char *>(g_slots),
+                   slot_bytes, lane);
+            x.slots = sslots;
+        } else {
+            x.slots = g_slots;
+        }
         x.tset = tset;
         __syncwarp();
         const long long o = p.offsets[r];
@@ -899,8 +926,7 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
         x.plen = p.plen + o;
         x.olen = p.olen + o;
         x.tier = p.tier + o;
-        x.g = p.g + o;
-        x.link = p.link + o;
+        x.node = p.node + o;
         x.res = p.res + o;
         x.log = p.log + (size_t)r * p.cap;
         x.magic = magic;
@@ -973,7 +999,7 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
                     x.t = bz[j];
                     tlast = max(tlast, bz[j]);
                     if (C > 1) fresh += tset_insert(x, bz[j]);
-                    if (inst_complete_head(x, cn, i)) pend |= 1u << j;
+                    if (inst_complete_head(x, i)) pend |= 1u << j;
                     else inst_form(x, cn, i, p.base, p.a, p.b);
                 }
                 __syncwarp();
@@ -1071,6 +1097,9 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
             a_ev += __shfl_xor_sync(kFull, a_ev, sh);
         }
         copy16(gblob, blob, p.L.bytes, lane);
+        if (SMS)
+            copy16(reinterpret_cast<unsigned char *>(g_slots), reinterpret_cast<const unsigned char *>(sslots),
+                   slot_bytes, lane);
         if (l0) {
             RepState o2;
             o2.t = x.t;
@@ -1120,8 +1149,6 @@ __global__ void k_init_state(Params p, const int *rep_table, const int *tbl_k, c
             b[L.nrun + i] = 0;
             b[L.pc + i] = 0;
             b[L.phase + i] = 0;
-            b[L.alo + i] = 0;
-            b[L.ahi + i] = 0;
             b[L.mrole + i] = MIG_NONE;
             b[L.mpeer + i] = 0;
         }
@@ -1130,6 +1157,7 @@ __global__ void k_init_state(Params p, const int *rep_table, const int *tbl_k, c
             reinterpret_cast<uint16_t *>(b + L.cnt)[i] = 0;
             reinterpret_cast<uint32_t *>(b + L.head)[i] = kNone;
             reinterpret_cast<uint32_t *>(b + L.tail)[i] = kNone;
+            reinterpret_cast<uint32_t *>(b + L.hinfo)[i] = 0;
         }
         for (int k = lane; k < p.K; k += 32)
             reinterpret_cast<int *>(b + L.h)[k] = k < K ? tbl_h[tb * p.K + k] : 0;
@@ -1143,11 +1171,9 @@ __global__ void k_init_state(Params p, const int *rep_table, const int *tbl_k, c
     }
 }
 
-__global__ void k_init_requests(sim_request_result_t *res, uint16_t *g, long long n) {
-    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
+__global__ void k_init_requests(sim_request_result_t *res, long long n) {
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x)
         reinterpret_cast<uint4 *>(res)[i] = make_uint4(0xFFFFFFFFu, kNone, kNone, 0u);
-        g[i] = 0;
-    }
 }
 
 // Trace validation: bit 0 unsorted, 1 tier >= K, 2 zero length, 3 too long, 4 bad arrival.
@@ -1196,12 +1222,13 @@ __global__ void k_export_stats(const RepState *rep, sim_replica_stats_t *out, in
 // ---- launch configuration ---------------------------------------------------
 typedef void (*RunKernel)(Params);
 
-inline RunKernel pick(int c) {  // c = instances per lane
+template <bool SMS>
+RunKernel pick(int c) {  // c = instances per lane
     switch (c) {
-        case 1: return k_run<1>;
-        case 2: return k_run<2>;
-        case 4: return k_run<4>;
-        default: return k_run<8>;
+        case 1: return k_run<1, SMS>;
+        case 2: return k_run<2, SMS>;
+        case 4: return k_run<4, SMS>;
+        default: return k_run<8, SMS>;
     }
 }
 
@@ -1236,14 +1263,13 @@ inline Layout make_layout(int N, int K, int T) {
     L.minfin = take(4u * N, 16);
     L.head = take(4u * N * K, 16);
     L.tail = take(4u * N * K, 16);
+    L.hinfo = take(4u * N * K, 16);
     L.h = take(4u * K, 16);
     L.wmask = take(2u * N, 16);
     L.cnt = take(2u * N * K, 16);
     L.nrun = take(N, 16);
     L.pc = take(N, 16);
     L.phase = take(N, 16);
-    L.alo = take(N, 16);
-    L.ahi = take(N, 16);
     L.mrole = take(N, 16);
     L.mpeer = take(N, 16);
     L.hist = take((uint32_t)N * hist_stride(T), 16);
@@ -1256,9 +1282,14 @@ inline Layout make_layout(int N, int K, int T) {
 inline uint32_t hash_bytes_for(int N) { return lanes_c(N) > 1 ? kHashSlots * 4u : 0u; }
 
 // Chooses the kernel variant and grid for a problem; cudaSuccess or the error.
-inline cudaError_t plan_launch(int R, int N, const Layout &L, Launch &out) {
-    out.fn = pick(lanes_c(N));
-    out.smem = kMagicBytes + (size_t)kWarpsPerBlock * (L.bytes + hash_bytes_for(N));
+// Running-request records go to shared memory while a replica's take at most this many bytes.
+constexpr uint32_t kSmemSlotLimit = 24u * 1024u;
+
+inline cudaError_t plan_launch(int R, int N, int Bmax, const Layout &L, Launch &out) {
+    const uint32_t slot_bytes = (uint32_t)N * (uint32_t)Bmax * 16u;
+    const bool sms = slot_bytes <= kSmemSlotLimit;
+    out.fn = sms ? pick<true>(lanes_c(N)) : pick<false>(lanes_c(N));
+    out.smem = kMagicBytes + (size_t)kWarpsPerBlock * (L.bytes + (sms ? slot_bytes : 0u) + hash_bytes_for(N));
     int dev = 0, sms_count = 0, per_sm = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms_count, cudaDevAttrMultiProcessorCount, dev);
@@ -1304,9 +1335,9 @@ struct sim {
     std::vector<int64_t> h_off;
     long long *d_off = nullptr;
     uint32_t *d_arrival = nullptr;
-    uint16_t *d_plen = nullptr, *d_olen = nullptr, *d_g = nullptr;
+    uint16_t *d_plen = nullptr, *d_olen = nullptr;
     uint8_t *d_tier = nullptr;
-    uint2 *d_link = nullptr;
+    uint4 *d_node = nullptr;
     sim_request_result_t *d_res = nullptr;
     int sms = 0;
     std::string err;
@@ -1394,8 +1425,7 @@ mt::Params make_params(const sim_t *s, long long max_steps) {
     p.plen = s->d_plen;
     p.olen = s->d_olen;
     p.tier = s->d_tier;
-    p.g = s->d_g;
-    p.link = s->d_link;
+    p.node = s->d_node;
     p.res = s->d_res;
     p.blobs = s->d_blobs;
     p.slots = s->d_slots;
@@ -1419,7 +1449,7 @@ int reset_state(sim_t *s) {
     if (rc) return rc;
     if (s->qtot > 0) {
         const long long nb = std::min<long long>((s->qtot + 255) / 256, 65535LL * 16);
-        mt::k_init_requests<<<(unsigned)nb, 256, 0, s->stream>>>(s->d_res, s->d_g, (long long)s->qtot);
+        mt::k_init_requests<<<(unsigned)nb, 256, 0, s->stream>>>(s->d_res, (long long)s->qtot);
         rc = check_launch(s, "k_init_requests");
     }
     return rc;
@@ -1543,7 +1573,8 @@ int sim_create(const sim_cluster_t *cl, const sim_tier_table_t *tt, const sim_po
     int dev = 0;
     if (e == cudaSuccess) e = cudaGetDevice(&dev);
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&s->sms, cudaDevAttrMultiProcessorCount, dev);
-    if (e == cudaSuccess) e = mt::plan_launch(cl->num_replicas, cl->num_instances, s->L, s->launch);
+    if (e == cudaSuccess)
+        e = mt::plan_launch(cl->num_replicas, cl->num_instances, cl->max_batch, s->L, s->launch);
     if (e != cudaSuccess) {
         cudaGetLastError();
         rc = e == cudaErrorInvalidConfiguration
@@ -1572,19 +1603,18 @@ int sim_load_trace(sim_t *s, const int64_t *off, const uint32_t *arrival, const 
     s->loaded = false;
     if (n > s->qcap) {
         dfree(s, s->d_arrival); dfree(s, s->d_plen); dfree(s, s->d_olen); dfree(s, s->d_tier);
-        dfree(s, s->d_g); dfree(s, s->d_link); dfree(s, s->d_res);
-        s->d_arrival = nullptr; s->d_plen = s->d_olen = s->d_g = nullptr; s->d_tier = nullptr;
-        s->d_link = nullptr; s->d_res = nullptr;
+        dfree(s, s->d_node); dfree(s, s->d_res);
+        s->d_arrival = nullptr; s->d_plen = s->d_olen = nullptr; s->d_tier = nullptr;
+        s->d_node = nullptr; s->d_res = nullptr;
         s->qcap = -1;
         const size_t m = (size_t)std::max<int64_t>(n, 1);
         s->d_arrival = (uint32_t *)dalloc(s, m * 4);
         s->d_plen = (uint16_t *)dalloc(s, m * 2);
         s->d_olen = (uint16_t *)dalloc(s, m * 2);
         s->d_tier = (uint8_t *)dalloc(s, m);
-        s->d_g = (uint16_t *)dalloc(s, m * 2);
-        s->d_link = (uint2 *)dalloc(s, m * 8);
+        s->d_node = (uint4 *)dalloc(s, m * 16);
         s->d_res = (sim_request_result_t *)dalloc(s, m * 16);
-        if (!s->d_arrival || !s->d_plen || !s->d_olen || !s->d_tier || !s->d_g || !s->d_link || !s->d_res)
+        if (!s->d_arrival || !s->d_plen || !s->d_olen || !s->d_tier || !s->d_node || !s->d_res)
             return fail(s, SIM_ERR_OOM, "device allocation for %lld trace records failed", (long long)n);
         s->qcap = n;
     }
@@ -1749,8 +1779,7 @@ extern "C" int sim_run_static(const sim_cluster_t *cl, const sim_tier_table_t *t
     const size_t o_blobs = o; o = align256(o + (size_t)R * L.bytes);
     const size_t o_slots = o; o = align256(o + (size_t)R * N * cl->max_batch * 16);
     const size_t o_rep = o; o = align256(o + (size_t)R * sizeof(mt::RepState));
-    const size_t o_g = o; o = align256(o + (size_t)n * 2);
-    const size_t o_link = o; o = align256(o + (size_t)n * 8);
+    const size_t o_node = o; o = align256(o + (size_t)n * 16);
     const size_t o_off = o; o = align256(o + ((size_t)R + 1) * 8);
     const size_t o_rt = o; o = align256(o + (size_t)R * 4);
     const size_t o_tk = o; o = align256(o + (size_t)tt->num_tables * 4);
@@ -1775,7 +1804,7 @@ extern "C" int sim_run_static(const sim_cluster_t *cl, const sim_tier_table_t *t
     cudaStream_t st = (cudaStream_t)cuda_stream;
 
     mt::Launch lc;
-    e = mt::plan_launch(R, N, L, lc);
+    e = mt::plan_launch(R, N, cl->max_batch, L, lc);
     if (e != cudaSuccess) {
         cudaGetLastError();
         return e == cudaErrorInvalidConfiguration
@@ -1790,8 +1819,7 @@ extern "C" int sim_run_static(const sim_cluster_t *cl, const sim_tier_table_t *t
     p.plen = plen;
     p.olen = olen;
     p.tier = tier;
-    p.g = (uint16_t *)(base + o_g);
-    p.link = (uint2 *)(base + o_link);
+    p.node = (uint4 *)(base + o_node);
     p.res = per_request;
     p.blobs = base + o_blobs;
     p.slots = (uint4 *)(base + o_slots);
@@ -1827,7 +1855,7 @@ extern "C" int sim_run_static(const sim_cluster_t *cl, const sim_tier_table_t *t
     mt::k_init_state<<<(R + 7) / 8, 256, 0, st>>>(p, rt, tk, th);
     if (n > 0) {
         const long long nb = std::min<long long>((n + 255) / 256, 65535LL * 16);
-        mt::k_init_requests<<<(unsigned)nb, 256, 0, st>>>(per_request, p.g, (long long)n);
+        mt::k_init_requests<<<(unsigned)nb, 256, 0, st>>>(per_request, (long long)n);
     }
     lc.fn<<<lc.grid, 32 * mt::kWarpsPerBlock, lc.smem, st>>>(p);
     mt::k_export_stats<<<(R + 255) / 256, 256, 0, st>>>(p.rep, per_replica, R, nullptr);
