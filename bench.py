@@ -262,7 +262,7 @@ def bench_gpu(args):
             "replica_steps_per_gpu_step": int(steps_per_run),
             "parallelism": "replicas sharded across GPUs, no collective on the data path",
             "l2": "inputs larger than L2: trace %.0f MB + per-request state %.0f MB resident" % (
-                Q * 9 / 1e6, Q * 26 / 1e6),
+                Q * 9 / 1e6, Q * 32 / 1e6),
         },
         "request_events_per_s": tot_events / tot_s,
         "e2e": {"value": e2e_units / e2e_max, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},

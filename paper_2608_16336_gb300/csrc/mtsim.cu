@@ -12,12 +12,16 @@
 //   Instances are spread over lanes in contiguous blocks of C = ceil(N/32) per
 //   lane (C is a template parameter), so "lowest lane" order is "lowest
 //   instance" order.  Per-request state stays in HBM: the read-only trace
-//   (SoA), the 16-byte result record, the tokens generated so far and a doubly
-//   linked list node that threads waiting requests into their (instance, tier)
-//   FCFS bucket.  Running requests occupy per-instance slot arrays (request id
-//   + one packed 64-bit state word); a batch advance or batch formation touches
-//   an instance's slots as one 16-byte pair per lane.  The next 32 arrivals
-//   are held in registers, one per lane.
+//   (SoA), the 16-byte result record and a 16-byte queue node that threads a
+//   waiting request into its (instance, tier) FCFS bucket.  A running request
+//   is a 16-byte slot record that is written when it joins a batch and read
+//   only on events; batch advance is lazy (see the slot record below), so an
+//   iteration end and a batch formation without events cost O(1).
+//   Between global events (arrivals, migration ticks) the instances that are
+//   in no migration do not interact, so each lane advances its own instances
+//   through a window in which each ends at most one iteration; migrations and
+//   global events are stepped by the whole warp in the oracle's order.  The
+//   next 32 arrivals are held in registers, one per lane.
 //
 // Exactness
 //   Everything is integer.  Freeness F = (M - U) / max(B, 1) (Sec. 3.2 Eq. 1-2)
@@ -134,7 +138,7 @@ struct Params {
 };
 
 // Per-warp view of the replica being simulated: instance state in shared
-// memory, request state and slot records in HBM; scalars are warp-uniform
+// memory, request state in HBM, slot records in either; scalars are warp-uniform
 // except t while lanes advance their own instances.
 struct Ctx {
     uint32_t *busy, *mreq, *head, *tail, *hinfo, *nf, *minfin;
@@ -1278,7 +1282,7 @@ inline Layout make_layout(int N, int K, int T) {
     return L;
 }
 
-// Chooses the kernel variant and grid for a problem; cudaSuccess or the error.
+// Bytes of the per-warp event-time set; only variants with several instances per lane use it.
 inline uint32_t hash_bytes_for(int N) { return lanes_c(N) > 1 ? kHashSlots * 4u : 0u; }
 
 // Chooses the kernel variant and grid for a problem; cudaSuccess or the error.
