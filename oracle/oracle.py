@@ -26,7 +26,7 @@ SO = os.path.join(LIB_DIR, "liboracle.so")
 MAXK = 16
 NONE32 = 0xFFFFFFFF
 STATUS_DONE, STATUS_INCOMPLETE = 0, 1
-EV_QUEUED, EV_START, EV_COMMIT, EV_ABORT = 0, 1, 2, 3
+EV_QUEUED, EV_START, EV_COMMIT, EV_ABORT, EV_SCALE_OUT, EV_SCALE_IN = 0, 1, 2, 3, 4, 5
 
 
 class OracleConfig(ctypes.Structure):
@@ -46,7 +46,12 @@ class OracleConfig(ctypes.Structure):
         ("theta_num", ctypes.c_int32),
         ("theta_den", ctypes.c_int32),
         ("check_invariants", ctypes.c_int32),
+        ("autoscale", ctypes.c_int32),
+        ("scale_out_num", ctypes.c_int32),
+        ("scale_in_num", ctypes.c_int32),
+        ("scale_den", ctypes.c_int32),
         ("pad_", ctypes.c_int32),
+        ("drain_start_us", ctypes.c_void_p),
     ]
 
 
@@ -64,6 +69,8 @@ class OracleStats(ctypes.Structure):
         ("finished", ctypes.c_int64),
         ("last_time", ctypes.c_uint32),
         ("status", ctypes.c_int32),
+        ("scale_out_signals", ctypes.c_int64),
+        ("scale_in_signals", ctypes.c_int64),
     ]
 
 
@@ -129,7 +136,10 @@ def lib(so_path: str | None = None) -> ctypes.CDLL:
 def make_config(num_instances, blocks_per_instance, headroom, *, tokens_per_block=16, max_batch=64,
                 iter_base_us=4000, iter_us_per_prefill_token=20, iter_us_per_decode_seq=30,
                 migrate_blocks_per_iter=64, enable_migration=1, migrate_interval_us=50_000,
-                theta_num=3, theta_den=10, check_invariants=0) -> OracleConfig:
+                theta_num=3, theta_den=10, check_invariants=0, autoscale=0, scale_out_num=-1, scale_in_num=3,
+                scale_den=2, drain_start_us=None) -> OracleConfig:
+    """A replica's configuration; ``drain_start_us`` ([num_instances] times,
+    NONE32 = never) is kept alive on the returned object as ``_drain``."""
     c = OracleConfig()
     c.num_instances = num_instances
     c.blocks_per_instance = blocks_per_instance
@@ -147,6 +157,16 @@ def make_config(num_instances, blocks_per_instance, headroom, *, tokens_per_bloc
     c.theta_num = theta_num
     c.theta_den = theta_den
     c.check_invariants = check_invariants
+    c.autoscale = autoscale
+    c.scale_out_num = scale_out_num
+    c.scale_in_num = scale_in_num
+    c.scale_den = scale_den
+    c._drain = None
+    if drain_start_us is not None:
+        c._drain = np.ascontiguousarray(drain_start_us, np.uint32)
+        if c._drain.shape != (num_instances,):
+            raise ValueError("drain_start_us needs one time per instance")
+        c.drain_start_us = c._drain.ctypes.data
     return c
 
 
@@ -157,7 +177,10 @@ def config_for(w, r: int, check_invariants: int = 0) -> OracleConfig:
         iter_us_per_prefill_token=w.iter_us_per_prefill_token, iter_us_per_decode_seq=w.iter_us_per_decode_seq,
         migrate_blocks_per_iter=w.migrate_blocks_per_iter, enable_migration=w.enable_migration,
         migrate_interval_us=w.migrate_interval_us, theta_num=w.theta_num, theta_den=w.theta_den,
-        check_invariants=check_invariants)
+        check_invariants=check_invariants, autoscale=getattr(w, "autoscale", 0),
+        scale_out_num=getattr(w, "scale_out_num", -1), scale_in_num=getattr(w, "scale_in_num", 3),
+        scale_den=getattr(w, "scale_den", 2),
+        drain_start_us=None if getattr(w, "drain_start_us", None) is None else w.drain_start_us[r])
 
 
 class ReplicaResult:
@@ -226,7 +249,9 @@ def run_workload(w, replicas=None, *, nthreads: int = 1, max_steps: int = 1 << 6
         res = ReplicaResult(sl.stop - sl.start, log_capacity)
         io, k = _io_for(w.arrival_us[sl], w.prompt_len[sl], w.output_len[sl], w.tier[sl], res)
         keep.append(k)
-        cfgs[j] = config_for(w, r, check_invariants)
+        cfg = config_for(w, r, check_invariants)
+        keep.append(cfg._drain)
+        cfgs[j] = cfg
         ios[j] = io
         results[r] = res
     lib(so_path).oracle_run_many(n, cfgs, ios, max_steps, stats, nthreads)

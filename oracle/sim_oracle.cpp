@@ -29,6 +29,18 @@
  *    small-KV running request: each source iteration end copies up to S
  *    blocks; the request commits to the destination when all of its blocks
  *    are copied.
+ *  - Draining (Sec. 3.4, Sec. 3.5, the last case of Eq. 2): from its drain
+ *    start time on, an instance's virtual usage is infinite.  It gets no
+ *    dispatch unless every instance drains (then the least loaded draining
+ *    one, by ordinary freeness, gets it), it is the first migration source at
+ *    every tick (no threshold: its freeness is minus infinity) and never a
+ *    destination.  Its own batches keep running.
+ *  - Auto-scaling signal (Sec. 3.4, Sec. 3.6): at every tick, the mean of the
+ *    normal-priority freeness F_normal (Eq. 1 without the headroom term) over
+ *    the instances that are not draining is compared, exactly, with the
+ *    scale-out and scale-in thresholds (-1/2 and 3/2 in the paper); each
+ *    signal is counted and logged.  Nothing is added or removed: the signal
+ *    is an output.
  *  - Local scheduling (Sec. 2.2, Sec. 3.1): continuous batching with
  *    priority-ordered queues (one FCFS bucket per tier), block-level KV
  *    allocation (ceil((P+g)/T) blocks for P prompt and g generated tokens),
@@ -53,7 +65,7 @@ constexpr int MAXK = 16;
 
 enum Status { ST_DONE = 0, ST_INCOMPLETE = 1, ST_ARG = -1, ST_TRACE = -2, ST_OVERFLOW = -5,
               ST_INVARIANT = -9, ST_DEADLOCK = -10 };
-enum EvKind { EV_QUEUED = 0, EV_START = 1, EV_COMMIT = 2, EV_ABORT = 3 };
+enum EvKind { EV_QUEUED = 0, EV_START = 1, EV_COMMIT = 2, EV_ABORT = 3, EV_SCALE_OUT = 4, EV_SCALE_IN = 5 };
 enum ReqState { PENDING = 0, WAITING = 1, RUNNING = 2, DONE = 3 };
 enum MigRole { MIG_NONE = 0, MIG_SRC = 1, MIG_DST = 2 };
 
@@ -74,7 +86,10 @@ typedef struct {
     int64_t migrate_interval_us;
     int32_t theta_num, theta_den;
     int32_t check_invariants;
+    int32_t autoscale;               /* evaluate the auto-scaling signal at every tick */
+    int32_t scale_out_num, scale_in_num, scale_den;  /* thresholds on the mean F_normal */
     int32_t pad_;
+    const uint32_t *drain_start_us;  /* [num_instances] or NULL: instance i drains from that time on */
 } oracle_config_t;
 
 typedef struct {
@@ -90,6 +105,8 @@ typedef struct {
     int64_t finished;
     uint32_t last_time;
     int32_t status;
+    int64_t scale_out_signals;   /* ticks at which the mean F_normal was below the scale-out threshold */
+    int64_t scale_in_signals;    /* ticks at which it was above the scale-in threshold */
 } oracle_stats_t;
 
 typedef struct {
@@ -173,6 +190,18 @@ struct Sim {
         num = (int64_t)c.blocks_per_instance - usage;
         den = in.running.empty() ? 1 : (int64_t)in.running.size();
     }
+    /* Normal-priority freeness (Sec. 3.4): the same fraction without the headroom term. */
+    void normal_freeness(const Inst &in, int64_t &num, int64_t &den) const {
+        int64_t usage = 0;
+        for (int r : in.running) usage += req[r].blocks;
+        int h = hol_request(in);
+        if (h >= 0) usage += need_blocks(req[h]);
+        usage += in.reserved_in;
+        num = (int64_t)c.blocks_per_instance - usage;
+        den = in.running.empty() ? 1 : (int64_t)in.running.size();
+    }
+    /* An instance drains from its drain start time on (Sec. 3.5). */
+    bool draining(int i) const { return c.drain_start_us != nullptr && now >= c.drain_start_us[i]; }
     /* true when F_a > F_b */
     bool freer(int a, int b) const {
         int64_t na, da, nb, db;
@@ -301,9 +330,12 @@ struct Sim {
         while (cursor < io.nreq && io.arrival_us[cursor] == now) arr.push_back((int)cursor++);
         std::stable_sort(arr.begin(), arr.end(), [&](int a, int b) { return req[a].tier < req[b].tier; });
         for (int r : arr) {
-            int best = 0;
-            for (int i = 1; i < c.num_instances; ++i)
-                if (freer(i, best)) best = i;
+            int best = -1;  /* freest instance that is not draining, lowest index on ties */
+            for (int i = 0; i < c.num_instances; ++i)
+                if (!draining(i) && (best < 0 || freer(i, best))) best = i;
+            if (best < 0)   /* every instance drains: the least loaded of them */
+                for (int i = 0; i < c.num_instances; ++i)
+                    if (best < 0 || freer(i, best)) best = i;
             Req &q = req[r];
             inst[best].waiting[q.tier].push_back(r);
             inst[best].cnt[q.tier]++;
@@ -323,17 +355,26 @@ struct Sim {
             n_el += eligible[i];
         }
         while (n_el >= 2) {
+            /* A draining instance has infinite virtual usage, so it is the least free
+             * (lowest index among several) and passes the threshold against any other. */
             int s = -1;
             for (int i = 0; i < c.num_instances; ++i)
-                if (eligible[i] && (s < 0 || freer(s, i))) s = i;     /* least free, lowest index */
+                if (eligible[i] && draining(i)) { s = i; break; }
+            const bool drain_source = s >= 0;
+            if (!drain_source)
+                for (int i = 0; i < c.num_instances; ++i)
+                    if (eligible[i] && (s < 0 || freer(s, i))) s = i;     /* least free, lowest index */
             int d = -1;
             for (int i = 0; i < c.num_instances; ++i)
-                if (eligible[i] && i != s && (d < 0 || freer(i, d))) d = i;  /* freest, lowest index */
-            int64_t ns, ds, nd, dd;
-            freeness(inst[s], ns, ds);
-            freeness(inst[d], nd, dd);
-            /* F_d - F_s >= theta_num / theta_den, exactly */
-            if ((int64_t)c.theta_den * (nd * ds - ns * dd) < (int64_t)c.theta_num * dd * ds) break;
+                if (eligible[i] && i != s && !draining(i) && (d < 0 || freer(i, d))) d = i;  /* freest, lowest index */
+            if (d < 0) break;  /* nothing but draining instances left to receive */
+            if (!drain_source) {
+                int64_t ns, ds, nd, dd;
+                freeness(inst[s], ns, ds);
+                freeness(inst[d], nd, dd);
+                /* F_d - F_s >= theta_num / theta_den, exactly */
+                if ((int64_t)c.theta_den * (nd * ds - ns * dd) < (int64_t)c.theta_num * dd * ds) break;
+            }
             Inst &S = inst[s];
             Inst &D = inst[d];
             bool moved = false;
@@ -377,6 +418,44 @@ struct Sim {
             eligible[s] = false;
             --n_el;
             if (moved) { eligible[d] = false; --n_el; }
+        }
+    }
+
+    /* Auto-scaling signal at a tick (Sec. 3.6).  The mean is kept as an exact
+     * fraction p/q (q > 0, reduced): every F_normal has a denominator of at
+     * most Bmax, so q divides lcm(1..Bmax) < 2^91 and 128-bit integers hold
+     * every product below. */
+    static __int128 gcd128(__int128 a, __int128 b) {
+        if (a < 0) a = -a;
+        while (b != 0) {
+            __int128 t = a % b;
+            a = b;
+            b = t;
+        }
+        return a;
+    }
+    void phase_autoscale() {
+        __int128 p = 0, q = 1;
+        int64_t n = 0;
+        for (int i = 0; i < c.num_instances; ++i) {
+            if (draining(i)) continue;  /* an instance that is leaving does not count */
+            int64_t num, den;
+            normal_freeness(inst[i], num, den);
+            p = p * den + (__int128)num * q;
+            q = q * den;
+            __int128 g = gcd128(p, q);
+            p /= g;
+            q /= g;
+            ++n;
+        }
+        if (n == 0) return;
+        /* mean = p / (q n) against threshold x / scale_den  <=>  p * scale_den against x * n * q */
+        if (p * c.scale_den < (__int128)c.scale_out_num * n * q) {
+            st.scale_out_signals++;
+            log_event(EV_SCALE_OUT, -1, 255, 255, 0);
+        } else if (p * c.scale_den > (__int128)c.scale_in_num * n * q) {
+            st.scale_in_signals++;
+            log_event(EV_SCALE_IN, -1, 255, 255, 0);
         }
     }
 
@@ -496,6 +575,10 @@ struct Sim {
         if (c.num_tiers < 1 || c.num_tiers > MAXK || c.migrate_blocks_per_iter < 1) return false;
         if (c.migrate_interval_us < 1 || c.theta_den < 1 || c.theta_num < 0) return false;
         if (c.iter_base_us < 0 || c.iter_us_per_prefill_token < 0 || c.iter_us_per_decode_seq < 0) return false;
+        if (c.autoscale != 0 && c.autoscale != 1) return false;
+        if (c.autoscale && (c.scale_den < 1 || c.scale_den > 64 || c.scale_out_num >= c.scale_in_num ||
+                            c.scale_out_num < -4096 || c.scale_in_num > 4096 || c.max_batch > 64))
+            return false;
         for (int k = 0; k < c.num_tiers; ++k)
             if (c.headroom[k] < 0) return false;
         return true;
@@ -544,7 +627,7 @@ struct Sim {
                 if (in.busy) t = std::min<int64_t>(t, in.busy_until);
             if (t == INF) { st.status = ST_DEADLOCK; return; }
             bool tick = false;
-            if (c.enable_migration && next_tick <= t) { t = next_tick; tick = true; }
+            if ((c.enable_migration || c.autoscale) && next_tick <= t) { t = next_tick; tick = true; }
             now = (uint32_t)t;
             st.steps++;
             st.last_time = now;
@@ -552,7 +635,8 @@ struct Sim {
             phase_dispatch();
             if (tick) {
                 next_tick += c.migrate_interval_us;
-                phase_migration_tick();
+                if (c.autoscale) phase_autoscale();
+                if (c.enable_migration) phase_migration_tick();
             }
             if (!phase_batch_formation()) { st.status = ST_INVARIANT; return; }
             if (st.status == ST_OVERFLOW) return;

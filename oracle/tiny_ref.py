@@ -8,6 +8,13 @@ Eq. 4), explicit batch-membership sets, and selections made with ``min``/
 ``max`` over explicit keys.  Only for a handful of instances and a few dozen
 requests.
 
+Draining (Sec. 3.5, the last case of Eq. 2) is the literal sentinel: the
+freeness of a draining instance is minus infinity, so comparisons do the
+rest; only the dispatch fallback when every instance drains (Sec. 3.4) looks
+at ordinary freeness.  The auto-scaling signal (Sec. 3.6) averages the
+normal-priority freeness, a ``Fraction`` without the headroom term, over the
+instances that are not draining.
+
 ``binary=True`` replaces the per-tier table by the original two-class
 Llumnix rule quoted in Sec. 3.3: every high-priority request (tier 0) present
 on an instance carries headroom h / numHighPriorityRequests and every other
@@ -18,7 +25,8 @@ from __future__ import annotations
 from fractions import Fraction
 
 NONE32 = 0xFFFFFFFF
-QUEUED, START, COMMIT, ABORT = 0, 1, 2, 3
+QUEUED, START, COMMIT, ABORT, SCALE_OUT, SCALE_IN = 0, 1, 2, 3, 4, 5
+MINUS_INF = float("-inf")
 
 
 def _ceil_div(a: int, b: int) -> int:
@@ -27,13 +35,17 @@ def _ceil_div(a: int, b: int) -> int:
 
 class TinySim:
     def __init__(self, n, m, headroom, trace, *, t_blk=16, bmax=64, base=4000, a=20, b=30, s_blocks=64,
-                 migration=True, interval=50_000, theta=Fraction(3, 10), binary=False, binary_h=0):
+                 migration=True, interval=50_000, theta=Fraction(3, 10), binary=False, binary_h=0,
+                 drain=None, autoscale=False, scale_out=Fraction(-1, 2), scale_in=Fraction(3, 2)):
         self.N, self.M, self.T, self.Bmax = n, m, t_blk, bmax
         self.H = list(headroom)
         self.K = len(self.H)
         self.base, self.a, self.b, self.S = base, a, b, s_blocks
         self.migration, self.interval, self.theta = migration, interval, theta
         self.binary, self.binary_h = binary, binary_h
+        self.drain = list(drain) if drain is not None else [NONE32] * n
+        self.autoscale, self.scale_out, self.scale_in = autoscale, scale_out, scale_in
+        self.signals = {"out": 0, "in": 0}
         self.trace = [tuple(int(x) for x in rec) for rec in trace]   # (arrival, P, O, tier)
         q = len(self.trace)
         self.g = [0] * q
@@ -86,8 +98,21 @@ class TinySim:
         total += self.reserved[i]
         return total
 
-    def F(self, i):
+    def draining(self, i):
+        return self.now >= self.drain[i]
+
+    def F_plain(self, i):
         return (self.M - self.virtual_usage(i)) / max(len(self.running[i]), 1)
+
+    def F(self, i):
+        """F_full with the drain sentinel: infinite usage, minus infinite freeness."""
+        return MINUS_INF if self.draining(i) else self.F_plain(i)
+
+    def F_normal(self, i):
+        h = self.hol(i)
+        used = sum(self.blocks[r] for r in self.running[i]) + (self.demand(h) if h is not None else 0)
+        used += self.reserved[i]
+        return Fraction(self.M - used, max(len(self.running[i]), 1))
 
     def dst_of(self, i):
         for s, mg in self.mig.items():
@@ -147,6 +172,8 @@ class TinySim:
     def _dispatch(self, arrivals):
         for r in sorted(arrivals, key=lambda x: (self.trace[x][3], x)):
             best = max(range(self.N), key=lambda i: (self.F(i), -i))
+            if self.F(best) == MINUS_INF:   # all draining: the least loaded of them
+                best = max(range(self.N), key=lambda i: (self.F_plain(i), -i))
             self.queues[best][self.trace[r][3]].append(r)
             self.loc[r] = ("wait", best)
             self.out["dispatch"][r] = best
@@ -158,7 +185,7 @@ class TinySim:
             fs = {i: self.F(i) for i in pool}
             s = min(pool, key=lambda i: (fs[i], i))
             d = max((i for i in pool if i != s), key=lambda i: (fs[i], -i))
-            if fs[d] - fs[s] < self.theta:
+            if fs[d] == MINUS_INF or fs[d] - fs[s] < self.theta:
                 break
             moved = False
             tiers = [k for k in range(self.K) if self.queues[s][k]]
@@ -179,6 +206,18 @@ class TinySim:
             pool.remove(s)
             if moved:
                 pool.remove(d)
+
+    def _autoscale(self):
+        live = [i for i in range(self.N) if not self.draining(i)]
+        if not live:
+            return
+        mean = sum(self.F_normal(i) for i in live) / len(live)
+        if mean < self.scale_out:
+            self.signals["out"] += 1
+            self.log.append((self.now, NONE32, 255, 255, 0, SCALE_OUT))
+        elif mean > self.scale_in:
+            self.signals["in"] += 1
+            self.log.append((self.now, NONE32, 255, 255, 0, SCALE_IN))
 
     def _form(self, i):
         if self.busy_until[i] is not None:
@@ -236,7 +275,7 @@ class TinySim:
             if not cands:
                 raise RuntimeError("deadlock")
             t = min(cands)
-            do_tick = self.migration and tick <= t
+            do_tick = (self.migration or self.autoscale) and tick <= t
             if do_tick:
                 t = tick
             self.now = t
@@ -251,7 +290,10 @@ class TinySim:
             self._dispatch(arrivals)
             if do_tick:
                 tick += self.interval
-                self._tick()
+                if self.autoscale:
+                    self._autoscale()
+                if self.migration:
+                    self._tick()
             for i in range(self.N):
                 self._form(i)
         return self

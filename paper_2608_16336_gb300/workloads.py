@@ -164,6 +164,14 @@ class Workload:
     theta_num: int = 3
     theta_den: int = 10
     enable_migration: int = 1
+    # auto-scaling signal (Sec. 3.6): thresholds on the mean F_normal, scale_out_num/scale_den
+    # and scale_in_num/scale_den (the paper's -1/2 and 3/2)
+    autoscale: int = 0
+    scale_out_num: int = -1
+    scale_in_num: int = 3
+    scale_den: int = 2
+    # drain schedule (Sec. 3.5): uint32 [R, N] start times, 0xFFFFFFFF = never; None = no draining
+    drain_start_us: np.ndarray = field(default=None)
     # trace (concatenated SoA, replica r owns [offsets[r], offsets[r+1]))
     offsets: np.ndarray = field(default=None)   # int64 [R+1]
     arrival_us: np.ndarray = field(default=None)
@@ -206,6 +214,9 @@ class Workload:
             iter_us_per_decode_seq=self.iter_us_per_decode_seq,
             migrate_blocks_per_iter=self.migrate_blocks_per_iter, migrate_interval_us=self.migrate_interval_us,
             theta_num=self.theta_num, theta_den=self.theta_den, enable_migration=self.enable_migration,
+            autoscale=self.autoscale, scale_out_num=self.scale_out_num, scale_in_num=self.scale_in_num,
+            scale_den=self.scale_den,
+            drain_start_us=None if self.drain_start_us is None else self.drain_start_us[idx].copy(),
             offsets=off, arrival_us=self.arrival_us[sel], prompt_len=self.prompt_len[sel],
             output_len=self.output_len[sel], tier=self.tier[sel],
             labels=[self.labels[r] for r in idx] if self.labels else [],

@@ -6,14 +6,18 @@ import numpy as np
 import pytest
 
 from oracle import oracle as O
+from tests import test_oracle_autoscale as apins
 from tests import test_oracle_pins as pins
 
 MUTANTS = {
-    "drop HoL demand (Eq. 2)": ("if (h >= 0) usage += need_blocks(req[h]);", "(void)h;"),
+    "drop HoL demand (Eq. 2)": ("if (h >= 0) usage += need_blocks(req[h]);                      /* HoL demand",
+                                "(void)h;  /* HoL demand"),
     "headroom per request instead of per tier (Eq. 4)": (
         "if (in.cnt[k] > 0) usage += c.headroom[k];", "usage += (int64_t)c.headroom[k] * in.cnt[k];"),
-    "drop inbound reservation": ("usage += in.reserved_in;", ""),
-    "dispatch ties to highest index": ("if (freer(i, best)) best = i;", "if (!freer(best, i)) best = i;"),
+    "drop inbound reservation": ("usage += in.reserved_in;                                       /* inbound",
+                                 "/* inbound"),
+    "dispatch ties to highest index": ("if (!draining(i) && (best < 0 || freer(i, best))) best = i;",
+                                       "if (!draining(i) && (best < 0 || !freer(best, i))) best = i;"),
     "migration gate sign flipped": ("(nd * ds - ns * dd) <", "(ns * dd - nd * ds) <"),
     "oldest preemption victim": ("(req[x].tier == req[v].tier && x > v)", "(req[x].tier == req[v].tier && x < v)"),
     "queued candidate from the front": ("int r = S.waiting[kq].back();\n                S.waiting[kq].pop_back();",
@@ -22,17 +26,43 @@ MUTANTS = {
         "c.iter_us_per_prefill_token * prefill_tokens +\n                              c.iter_us_per_decode_seq * n_decode",
         "c.iter_us_per_decode_seq * prefill_tokens +\n                              c.iter_us_per_prefill_token * n_decode"),
     "stage ignores destination memory": ("if (d.free_blocks < c_blocks) { abort_migration(si); return; }", ""),
-    "batch size counted from zero": ("den = in.running.empty() ? 1 : (int64_t)in.running.size();",
-                                     "den = (int64_t)in.running.size() + 1;"),
+    "batch size counted from zero": (
+        "/* inbound migration copy */\n        num = (int64_t)c.blocks_per_instance - usage;\n"
+        "        den = in.running.empty() ? 1 : (int64_t)in.running.size();",
+        "/* inbound migration copy */\n        num = (int64_t)c.blocks_per_instance - usage;\n"
+        "        den = (int64_t)in.running.size() + 1;"),
     "KV need rounds down": ("return (r.P + r.g + c.tokens_per_block - 1) / c.tokens_per_block;",
                             "return (r.P + r.g) / c.tokens_per_block;"),
+    "F_normal keeps the headroom": (
+        "        usage += in.reserved_in;\n        num = (int64_t)c.blocks_per_instance - usage;\n"
+        "        den = in.running.empty() ? 1 : (int64_t)in.running.size();\n    }\n    /* An instance drains",
+        "        usage += in.reserved_in;\n        for (int k = 0; k < c.num_tiers; ++k) if (in.cnt[k] > 0) "
+        "usage += c.headroom[k];\n        num = (int64_t)c.blocks_per_instance - usage;\n"
+        "        den = in.running.empty() ? 1 : (int64_t)in.running.size();\n    }\n    /* An instance drains"),
+    "mean over draining instances too": ("if (draining(i)) continue;  /* an instance that is leaving", "/* leaving"),
+    "scale-in threshold not strict": ("} else if (p * c.scale_den > (__int128)c.scale_in_num * n * q) {",
+                                      "} else if (p * c.scale_den >= (__int128)c.scale_in_num * n * q) {"),
+    "scale-out threshold not strict": ("if (p * c.scale_den < (__int128)c.scale_out_num * n * q) {",
+                                       "if (p * c.scale_den <= (__int128)c.scale_out_num * n * q) {"),
+    "draining instance still gets dispatch": ("if (!draining(i) && (best < 0 || freer(i, best))) best = i;",
+                                              "if (best < 0 || freer(i, best)) best = i;"),
+    "fallback picks the lowest index": ("                    if (best < 0 || freer(i, best)) best = i;",
+                                        "                    if (best < 0) best = i;"),
+    "draining source needs the threshold": ("            if (!drain_source) {\n                int64_t ns",
+                                            "            {\n                int64_t ns"),
+    "draining instance as destination": ("if (eligible[i] && i != s && !draining(i) && (d < 0 || freer(i, d))) d = i;",
+                                         "if (eligible[i] && i != s && (d < 0 || freer(i, d))) d = i;"),
+    "drain starts one tick late": ("return c.drain_start_us != nullptr && now >= c.drain_start_us[i];",
+                                   "return c.drain_start_us != nullptr && now > c.drain_start_us[i];"),
 }
 
 
 def _pins_fail(so_path):
     failures = 0
     for check in (lambda: pins.check_tiny_agreement(range(120), so_path=so_path),
-                  lambda: _closed_forms(so_path)):
+                  lambda: _closed_forms(so_path),
+                  lambda: apins.check_tiny_drain_agreement(range(200), so_path=so_path),
+                  lambda: _autoscale_closed_form(so_path)):
         try:
             check()
         except AssertionError:
@@ -47,6 +77,15 @@ def _closed_forms(so_path):
                           np.array([1], np.uint8), so_path=so_path)
         assert int(res.first_token_us[0]) - 1000 == 4000 + 20 * P
         assert int(res.finish_us[0]) - int(res.first_token_us[0]) == (Ob - 1) * 4030
+
+
+def _autoscale_closed_form(so_path):
+    tr = (np.zeros(4, np.uint32), np.full(4, apins.P, np.uint16), np.full(4, apins.OUT, np.uint16),
+          np.zeros(4, np.uint8))
+    cfg = O.make_config(2, apins.M, [0], max_batch=1, enable_migration=0, autoscale=1)
+    res = O.run_trace(cfg, *tr, so_path=so_path)
+    assert apins._signals(res) == ([50_000, 100_000, 150_000, 200_000],
+                                   [250_000, 300_000, 350_000, 450_000, 500_000, 550_000, 600_000])
 
 
 @pytest.mark.parametrize("name", sorted(MUTANTS))
