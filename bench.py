@@ -214,8 +214,8 @@ def bench_gpu(args):
     pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
     h_arr, h_p, h_o, h_t = (pin(w.arrival_us.view(np.int32)), pin(w.prompt_len.view(np.int16)),
                             pin(w.output_len.view(np.int16)), pin(w.tier))
-    h_res = torch.empty(Q * 16, dtype=torch.uint8).pin_memory()
-    h_st = torch.empty(R * 64, dtype=torch.uint8).pin_memory()
+    h_res = torch.empty(Q * mtsim.RESULT_DTYPE.itemsize, dtype=torch.uint8).pin_memory()
+    h_st = torch.empty(R * mtsim.STATS_DTYPE.itemsize, dtype=torch.uint8).pin_memory()
     off = np.ascontiguousarray(w.offsets, np.int64)
 
     def e2e_step():
@@ -234,7 +234,7 @@ def bench_gpu(args):
     barrier()
     e2e_s = (time.perf_counter() - e0) / args.e2e_steps
     h2d = int(off.nbytes + Q * 9)
-    d2h = int(Q * 16 + R * 64)
+    d2h = int(h_res.numel() + h_st.numel())
     sim.close()
 
     tot_s, tot_units, tot_events = aggregate(dev_s, steps_per_run * args.steps, events_per_run * args.steps)

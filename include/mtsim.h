@@ -15,9 +15,13 @@
  *      tier, each to the instance of highest freeness F (Sec. 3.4), where
  *      F = (M - sum_r V(r)) / B (Sec. 3.2 Eq. 1-2) and the virtual usage
  *      includes the per-tier headroom H_k of every tier present, charged once
- *      per tier (Sec. 3.3 Eq. 3-4);
- *   3. at every migration interval, pairing of low- and high-freeness
- *      instances while max F - min F >= theta (Sec. 3.5);
+ *      per tier (Sec. 3.3 Eq. 3-4); an instance that is draining (see
+ *      sim_set_drain) has infinite virtual usage and gets no request unless
+ *      every instance drains, then the freest of them does (Sec. 3.4-3.5);
+ *   3. at every interval ("tick"): the auto-scaling signal when enabled
+ *      (mean normal-priority freeness against two thresholds, Sec. 3.6), then
+ *      pairing of low- and high-freeness instances while max F - min F >=
+ *      theta, draining instances first and without the threshold (Sec. 3.5);
  *   4. batch formation at idle instances (continuous batching with
  *      priority-ordered queues, KV growth and preemption, Sec. 2.2, 3.1) under
  *      the integer iteration-time model base + a*prefill_tokens + b*decodes.
@@ -78,6 +82,9 @@ extern "C" {
 #define SIM_EV_START 1   /* staged copy of a running request began (blocks = its KV size) */
 #define SIM_EV_COMMIT 2  /* the request committed to the destination (blocks = its KV size) */
 #define SIM_EV_ABORT 3   /* staged copy abandoned (blocks = blocks copied so far) */
+/* Auto-scaling signal records (Sec. 3.6): request = SIM_NONE32, src = dst = 255, blocks = 0. */
+#define SIM_EV_SCALE_OUT 4  /* mean F_normal below the scale-out threshold at this tick */
+#define SIM_EV_SCALE_IN 5   /* mean F_normal above the scale-in threshold at this tick */
 
 #define SIM_NONE32 0xFFFFFFFFu  /* "not set" for 32-bit times */
 #define SIM_NONE16 0xFFFFu      /* "not set" for 16-bit instance ids */
@@ -112,7 +119,20 @@ typedef struct {
     int32_t migrate_blocks_per_iter;    /* S: KV blocks copied per source iteration, in [1, 65535] */
     int32_t theta_num, theta_den;       /* imbalance threshold theta = num/den (0.3 = 3/10) */
     int32_t event_log_capacity;         /* migration-log records kept per replica, in [0, 2^24] */
-    int64_t migrate_interval_us;        /* rebalancing period, in [1, 2^31] (50 ms in Sec. 3.5) */
+    int64_t migrate_interval_us;        /* tick period, in [1, 2^31] (50 ms in Sec. 3.5) */
+    /* Auto-scaling signal (Sec. 3.4, 3.6), evaluated at every tick when
+     * autoscale = 1: the mean over non-draining instances of the
+     * normal-priority freeness F_normal = (M - running KV - HoL demand -
+     * inbound reservation) / max(B, 1), i.e. Eq. 1 without the headroom
+     * term, is compared exactly with scale_out_num / scale_den (strictly
+     * below: scale-out) and scale_in_num / scale_den (strictly above:
+     * scale-in).  The paper's thresholds are -1/2 and 3/2.  The signal is
+     * reported (counters and log records); it adds or removes no instance.
+     * With autoscale = 1 ticks happen even when migration is off.
+     * autoscale = 0 ignores the three thresholds. */
+    int32_t autoscale;                  /* 0 or 1 */
+    int32_t scale_out_num, scale_in_num; /* in [-4096, 4096], scale_out_num < scale_in_num */
+    int32_t scale_den;                  /* in [1, 64] */
 } sim_policy_t;
 
 /* Per-request outcome, 16 bytes.  Times are microseconds from the replica's
@@ -140,6 +160,8 @@ typedef struct {
     uint32_t finished;           /* requests finished */
     uint32_t last_time_us;       /* time of the last processed step */
     int32_t status;              /* SIM_REPLICA_* or a negative SIM_ERR_* code */
+    uint32_t scale_out_signals;  /* ticks with a scale-out signal (Sec. 3.6) */
+    uint32_t scale_in_signals;   /* ticks with a scale-in signal */
 } sim_replica_stats_t;
 
 typedef struct {
@@ -171,8 +193,8 @@ typedef struct {
  * additionally M + sum_k H_k must stay below 2^19 for every table) and
  * copied.  cuda_stream is a cudaStream_t (NULL = legacy default stream);
  * allocator may be NULL.  Allocates the per-replica and per-instance state
- * (about (N * (40 + 10 * K) + N * Bmax * 12 + 16 * log capacity + 160) bytes
- * per replica).  On success *out receives the object and SIM_OK is returned;
+ * (about N * (67 + 14 * K + T) + N * Bmax * 16 + 16 * log capacity + 4 * K +
+ * 500 bytes per replica).  On success *out receives the object and SIM_OK is returned;
  * on failure *out is NULL and sim_last_error(NULL) describes the error. */
 int sim_create(const sim_cluster_t *cluster, const sim_tier_table_t *tiers, const sim_policy_t *policy,
                void *cuda_stream, const sim_allocator_t *allocator, sim_t **out);
@@ -192,6 +214,20 @@ int sim_load_trace(sim_t *sim, const int64_t *replica_offsets, const uint32_t *a
 
 /* Resets every replica of the loaded trace to t = 0 (asynchronous). */
 int sim_reset(sim_t *sim);
+
+/* Sets the drain schedule (Sec. 3.4-3.5; the last case of Eq. 2): instance i
+ * of replica r is draining at every step whose time is >=
+ * drain_start_us[r * N + i] (SIM_NONE32 = never).  A draining instance keeps
+ * running its own batches and queue, but its virtual usage is infinite: it
+ * receives no dispatch while some instance of its replica is not draining,
+ * it is the first migration source at every tick (no imbalance threshold)
+ * and never a destination, and it is left out of the auto-scaling mean.
+ * drain_start_us: [R * N] times, host or device per on_device, copied (a host
+ * buffer may be reused when the call returns); NULL removes the schedule.
+ * The schedule takes effect at the next sim_load_trace or sim_reset.
+ * Returns SIM_ERR_OOM if its device copy (4 * R * N bytes) cannot be
+ * allocated.  sim_run_static has no drain schedule. */
+int sim_set_drain(sim_t *sim, const uint32_t *drain_start_us, int on_device);
 
 /* Advances every unfinished replica by at most max_steps_per_replica steps
  * (>= 1) in one persistent kernel launch; a later call resumes where this one
@@ -247,7 +283,7 @@ size_t sim_device_bytes(const sim_t *sim);
  * (NULL = legacy default stream).
  *
  * Limits: the state of all replicas must fit in the scratch array, about
- * R * (N * (40 + 10 * K) + N * Bmax * 12 + 100) + 10 * total records bytes;
+ * R * (N * (67 + 14 * K + T) + N * Bmax * 16 + 600) + 16 * total records bytes;
  * a larger problem returns SIM_ERR_ARG with the size it needed.  The first
  * call on a device looks up the array's device address (cudaGetSymbolAddress)
  * with that device current, so make the first call before any stream capture.

@@ -96,7 +96,7 @@ constexpr uint32_t kFreshFlag = 1u << 8;  // set between admission and the end o
 // need no dependent HBM reads.
 
 struct Layout {
-    uint32_t busy, free_, resv, hol, hr, key, mreq, mcopied, nf, minfin;  // [N] x 4 B
+    uint32_t busy, free_, resv, hol, hr, key, mreq, mcopied, nf, minfin, drain;  // [N] x 4 B
     uint32_t wmask;                                                      // [N] x 2 B
     uint32_t nrun, pc, phase, mrole, mpeer;                               // [N] x 1 B
     uint32_t cnt;                                                        // [N*K] x 2 B
@@ -113,6 +113,7 @@ struct RepState {
     uint32_t next_tick, pad0;
     uint64_t steps, iterations, member_iterations, events;
     uint32_t migrations, preemptions, starts, aborts;
+    uint32_t scale_out, scale_in;
     int32_t status;
     uint32_t pad1;
 };
@@ -122,9 +123,14 @@ struct Params {
     uint32_t interval, max_steps;
     unsigned long long magT;      // ceil(2^40 / T)
     int base, a, b;
+    int ticks;                    // ticks happen (migration or the auto-scaling signal is on)
+    int autoscale, scale_out_num, scale_in_num, scale_den;
+    int drains;                   // a drain schedule is loaded
+    unsigned long long lcm_lo, lcm_hi;  // lcm(1, ..., Bmax) as two 64-bit halves
     Layout L;
     uint32_t hash_bytes;          // per-warp event-time set (C > 1 variants), else 0
     const long long *offsets;
+    const uint32_t *drain_src;    // [R][N] drain start times, or NULL
     const uint32_t *arrival;
     const uint16_t *plen, *olen;
     const uint8_t *tier;
@@ -141,7 +147,7 @@ struct Params {
 // memory, request state in HBM, slot records in either; scalars are warp-uniform
 // except t while lanes advance their own instances.
 struct Ctx {
-    uint32_t *busy, *mreq, *head, *tail, *hinfo, *nf, *minfin;
+    uint32_t *busy, *mreq, *head, *tail, *hinfo, *nf, *minfin, *drain;
     int *free_, *resv, *hol, *hr, *key, *mcopied, *h;
     uint16_t *wmask, *cnt;
     uint8_t *nrun, *pc, *phase, *mrole, *mpeer, *hist;
@@ -156,7 +162,7 @@ struct Ctx {
     sim_request_result_t *res;
     sim_migration_event_t *log;
     unsigned long long magT;
-    int N, K, T, TH, Bmax, S, cap, lane;
+    int N, K, T, TH, Bmax, S, cap, lane, drains;
     uint32_t Q, t;
 };
 
@@ -166,6 +172,7 @@ struct Ctx {
 // every window).
 struct Cnt {
     uint32_t finished, log_events, migrations, preemptions, starts, aborts, steps, iterations;
+    uint32_t scale_out, scale_in;  // lane 0 only
     uint64_t member_iterations, events;
     int status;
 };
@@ -647,11 +654,22 @@ __device__ __forceinline__ void arr_refill(const Ctx &x, ArrBuf &ab, uint32_t cu
 }
 
 // Phase 2: arrivals at t, tier 0 first, FCFS (trace order) within a tier.
-template <int C>
+// EXT: draining instances may exist.
+template <int C, bool EXT>
 __device__ __forceinline__ void dispatch_phase(const Ctx &x, Cnt &cn, uint32_t &cursor, uint32_t &next_arr,
                                                ArrBuf &ab) {
     refresh_keys<C>(x);
-    const uint32_t all = own_mask<C>(x);
+    uint32_t all = own_mask<C>(x);
+    if (EXT && x.drains) {
+        // Draining instances (infinite virtual usage, Sec. 3.5) get no
+        // dispatch unless every instance drains; then the freest of them
+        // does (Sec. 3.4: the least loaded draining one).
+        uint32_t live = 0;
+#pragma unroll
+        for (int j = 0; j < C; ++j)
+            if (((all >> j) & 1u) && x.drain[x.lane * C + j] > x.t) live |= 1u << j;
+        if (__any_sync(kFull, live != 0)) all = live;
+    }
     const uint32_t off = cursor - ab.pb;
     uint32_t eq = __ballot_sync(kFull, (uint32_t)x.lane >= off && ab.time == x.t);
     if ((eq >> 31) && off > 0) {
@@ -707,24 +725,80 @@ __device__ __forceinline__ void dispatch_phase(const Ctx &x, Cnt &cn, uint32_t &
     next_arr = __shfl_sync(kFull, ab.time, (int)(cursor - ab.pb));
 }
 
-// Phase 3: periodic rebalancing between low- and high-freeness instances (Sec. 3.5).
+// Auto-scaling signal at a tick (Sec. 3.6): the mean normal-priority freeness
+// (Eq. 1 without the headroom term, Sec. 3.4) over the instances that are not
+// draining, compared exactly with scale_out_num / scale_den and
+// scale_in_num / scale_den.  Each F_normal = (free - HoL) / max(B, 1) is scaled
+// by L = lcm(1, ..., Bmax), so S = L * sum F_normal is an exact 128-bit
+// integer (|S| < 2^117), and mean < x / D  <=>  S * D < x * n * L.  Collective.
 template <int C>
+__device__ __forceinline__ void autoscale_tick(const Ctx &x, Cnt &cn, const Params &p) {
+    const __int128 L = (__int128)(((unsigned __int128)p.lcm_hi << 64) | p.lcm_lo);
+    __int128 sum = 0;
+    int n = 0;
+#pragma unroll
+    for (int j = 0; j < C; ++j) {
+        const int i = x.lane * C + j;
+        if (i < x.N && !(x.drains && x.drain[i] <= x.t)) {
+            const int num = x.free_[i] - x.hol[i];
+            const int den = max((int)x.nrun[i], 1);
+            sum += (__int128)num * (L / den);
+            ++n;
+        }
+    }
+#pragma unroll
+    for (int sh = 16; sh > 0; sh >>= 1) {
+        const unsigned long long lo = __shfl_xor_sync(kFull, (unsigned long long)sum, sh);
+        const unsigned long long hi = __shfl_xor_sync(kFull, (unsigned long long)((unsigned __int128)sum >> 64), sh);
+        sum += (__int128)(((unsigned __int128)hi << 64) | lo);
+    }
+    n = __reduce_add_sync(kFull, n);
+    if (x.lane == 0 && n > 0) {
+        const __int128 lhs = sum * p.scale_den;
+        if (lhs < (__int128)p.scale_out_num * n * L) {
+            cn.scale_out++;
+            log_ev(x, cn, SIM_EV_SCALE_OUT, kNone, 255, 255, 0);
+        } else if (lhs > (__int128)p.scale_in_num * n * L) {
+            cn.scale_in++;
+            log_ev(x, cn, SIM_EV_SCALE_IN, kNone, 255, 255, 0);
+        }
+    }
+    __syncwarp();
+}
+
+// Phase 3: periodic rebalancing between low- and high-freeness instances (Sec. 3.5).
+template <int C, bool EXT>
 __device__ __forceinline__ void migration_tick(const Ctx &x, Cnt &cn, int theta_num, int theta_den) {
     refresh_keys<C>(x);
-    uint32_t el = 0;
+    uint32_t el = 0, dr = 0;  // eligible (not migrating); draining
 #pragma unroll
     for (int j = 0; j < C; ++j) {
         const int i = x.lane * C + j;
         if (i < x.N && x.mrole[i] == MIG_NONE) el |= 1u << j;
+        if (EXT && i < x.N && x.drains && x.drain[i] <= x.t) dr |= 1u << j;
     }
     for (;;) {
         const int nel = __reduce_add_sync(kFull, __popc(el));
         if (nel < 2) break;
-        const int s = arg_ext<C>(x, el, false, -1);
-        const int d = arg_ext<C>(x, el, true, s);
-        const long long ns = fnum(x, s), ds = max((int)x.nrun[s], 1);
-        const long long nd = fnum(x, d), dd = max((int)x.nrun[d], 1);
-        if ((long long)theta_den * (nd * ds - ns * dd) < (long long)theta_num * dd * ds) break;
+        // A draining instance has infinite virtual usage (Sec. 3.5): it is the
+        // least free (lowest index among several), passes the threshold
+        // against any other instance, and is never a destination.
+        int s;
+        const uint32_t dl = EXT ? __ballot_sync(kFull, (el & dr) != 0) : 0u;
+        if (dl) {
+            const int l = __ffs(dl) - 1;
+            const uint32_t bits = C == 1 ? 1u : __shfl_sync(kFull, el & dr, l);
+            s = l * C + __ffs(bits) - 1;
+        } else {
+            s = arg_ext<C>(x, el, false, -1);
+        }
+        const int d = arg_ext<C>(x, el & ~dr, true, s);
+        if (d < 0) break;
+        if (!dl) {
+            const long long ns = fnum(x, s), ds = max((int)x.nrun[s], 1);
+            const long long nd = fnum(x, d), dd = max((int)x.nrun[d], 1);
+            if ((long long)theta_den * (nd * ds - ns * dd) < (long long)theta_num * dd * ds) break;
+        }
         const bool has_wait = x.wmask[s] != 0;
         const int n_s = x.nrun[s];
         __syncwarp();
@@ -819,6 +893,7 @@ __device__ __forceinline__ void bind_blob(Ctx &x, const Layout &L, unsigned char
     x.mcopied = reinterpret_cast<int *>(blob + L.mcopied);
     x.nf = reinterpret_cast<uint32_t *>(blob + L.nf);
     x.minfin = reinterpret_cast<uint32_t *>(blob + L.minfin);
+    x.drain = reinterpret_cast<uint32_t *>(blob + L.drain);
     x.wmask = reinterpret_cast<uint16_t *>(blob + L.wmask);
     x.nrun = blob + L.nrun;
     x.pc = blob + L.pc;
@@ -889,8 +964,9 @@ __device__ __forceinline__ void form_all(const Ctx &x, Cnt &cn, uint32_t mask, c
 // every instance ends at most one iteration, and each lane advances its own
 // instances (an O(1) iteration end + batch formation); instances in a
 // migration, and every step at a global event, are advanced by lane 0 in the
-// oracle's order.
-template <int C, bool SMS>
+// oracle's order.  EXT: the variant that also handles draining instances and
+// the auto-scaling signal (the other variant compiles that code out).
+template <int C, bool SMS, bool EXT>
 __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
     extern __shared__ __align__(16) unsigned char smem[];
     unsigned long long *magic = reinterpret_cast<unsigned long long *>(smem);
@@ -943,6 +1019,7 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
         x.S = p.S;
         x.cap = p.cap;
         x.lane = lane;
+        x.drains = EXT ? p.drains : 0;
         x.t = rs.t;
         Cnt cn;  // lane 0: the replica's totals; other lanes: what they add in windows
         const bool l0 = lane == 0;
@@ -952,6 +1029,8 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
         cn.preemptions = l0 ? rs.preemptions : 0u;
         cn.starts = rs.starts;
         cn.aborts = rs.aborts;
+        cn.scale_out = rs.scale_out;
+        cn.scale_in = rs.scale_in;
         cn.steps = 0;
         cn.iterations = 0;
         cn.member_iterations = l0 ? rs.member_iterations : 0ull;
@@ -976,7 +1055,8 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
                 mb = min(mb, bz[j]);
             }
             const uint32_t tb = __reduce_min_sync(kFull, mb);
-            const uint32_t tg = p.enable_mig ? min(next_arr, next_tick) : next_arr;
+            const bool ticks = EXT ? p.ticks != 0 : p.enable_mig != 0;
+            const uint32_t tg = ticks ? min(next_arr, next_tick) : next_arr;
             if (tb < tg && max_steps - cn.steps > (uint32_t)x.N) {
                 // ---- window [tb, t1): at most one iteration end per instance ----
                 const uint32_t t1 =
@@ -1073,17 +1153,18 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
             // ---- one step at the next event time (global events, or near the step limit) ----
             const uint32_t tc = min(tb, next_arr);
             if (tc == kNone) { cn.status = SIM_ERR_DEADLOCK; break; }
-            const bool tick = p.enable_mig && next_tick <= tc;
+            const bool tick = ticks && next_tick <= tc;
             x.t = tick ? next_tick : tc;
             ++cn.steps;
             const uint32_t f1 = cn.finished;
             if (tb == x.t) complete_all<C>(x, cn, all);  // 1. iteration ends
             cn.finished = __shfl_sync(kFull, cn.finished, 0);
-            if (next_arr == x.t) dispatch_phase<C>(x, cn, cursor, next_arr, ab);  // 2. dispatch
-            if (tick) {  // 3. migration tick
+            if (next_arr == x.t) dispatch_phase<C, EXT>(x, cn, cursor, next_arr, ab);  // 2. dispatch
+            if (tick) {  // 3. auto-scaling signal and migration tick
                 const uint32_t nt = next_tick + p.interval;
                 next_tick = nt < next_tick ? kNone : nt;  // saturate: no tick beyond 2^32 - 1
-                migration_tick<C>(x, cn, p.theta_num, p.theta_den);
+                if (EXT && p.autoscale) autoscale_tick<C>(x, cn, p);
+                if (p.enable_mig) migration_tick<C, EXT>(x, cn, p.theta_num, p.theta_den);
             }
             form_all<C>(x, cn, all, p);  // 4. batch formation
             (void)f1;
@@ -1120,6 +1201,8 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
             o2.preemptions = cn.preemptions + a_pre;
             o2.starts = cn.starts;
             o2.aborts = cn.aborts;
+            o2.scale_out = cn.scale_out;
+            o2.scale_in = cn.scale_in;
             o2.status = cn.status;
             o2.pad1 = 0;
             p.rep[r] = o2;
@@ -1149,6 +1232,7 @@ __global__ void k_init_state(Params p, const int *rep_table, const int *tbl_k, c
             reinterpret_cast<int *>(b + L.mcopied)[i] = 0;
             reinterpret_cast<uint32_t *>(b + L.nf)[i] = 0;
             reinterpret_cast<uint32_t *>(b + L.minfin)[i] = kNone;
+            reinterpret_cast<uint32_t *>(b + L.drain)[i] = p.drain_src ? p.drain_src[(size_t)r * N + i] : kNone;
             reinterpret_cast<uint16_t *>(b + L.wmask)[i] = 0;
             b[L.nrun + i] = 0;
             b[L.pc + i] = 0;
@@ -1217,6 +1301,8 @@ __global__ void k_export_stats(const RepState *rep, sim_replica_stats_t *out, in
             o.finished = s.finished;
             o.last_time_us = s.t;
             o.status = s.status;
+            o.scale_out_signals = s.scale_out;
+            o.scale_in_signals = s.scale_in;
             out[r] = o;
         }
         if (unfinished && s.status != SIM_REPLICA_DONE) atomicAdd(unfinished, 1);
@@ -1226,19 +1312,21 @@ __global__ void k_export_stats(const RepState *rep, sim_replica_stats_t *out, in
 // ---- launch configuration ---------------------------------------------------
 typedef void (*RunKernel)(Params);
 
-template <bool SMS>
+template <bool SMS, bool EXT>
 RunKernel pick(int c) {  // c = instances per lane
     switch (c) {
-        case 1: return k_run<1, SMS>;
-        case 2: return k_run<2, SMS>;
-        case 4: return k_run<4, SMS>;
-        default: return k_run<8, SMS>;
+        case 1: return k_run<1, SMS, EXT>;
+        case 2: return k_run<2, SMS, EXT>;
+        case 4: return k_run<4, SMS, EXT>;
+        default: return k_run<8, SMS, EXT>;
     }
 }
 
+// fn / grid: the plain variant; fn_ext / grid_ext: the one with draining and
+// the auto-scaling signal (same shared memory).
 struct Launch {
-    RunKernel fn = nullptr;
-    int grid = 0;
+    RunKernel fn = nullptr, fn_ext = nullptr;
+    int grid = 0, grid_ext = 0;
     size_t smem = 0;
 };
 
@@ -1265,6 +1353,7 @@ inline Layout make_layout(int N, int K, int T) {
     L.mcopied = take(4u * N, 16);
     L.nf = take(4u * N, 16);
     L.minfin = take(4u * N, 16);
+    L.drain = take(4u * N, 16);
     L.head = take(4u * N * K, 16);
     L.tail = take(4u * N * K, 16);
     L.hinfo = take(4u * N * K, 16);
@@ -1292,20 +1381,25 @@ constexpr uint32_t kSmemSlotLimit = 24u * 1024u;
 inline cudaError_t plan_launch(int R, int N, int Bmax, const Layout &L, Launch &out) {
     const uint32_t slot_bytes = (uint32_t)N * (uint32_t)Bmax * 16u;
     const bool sms = slot_bytes <= kSmemSlotLimit;
-    out.fn = sms ? pick<true>(lanes_c(N)) : pick<false>(lanes_c(N));
+    out.fn = sms ? pick<true, false>(lanes_c(N)) : pick<false, false>(lanes_c(N));
+    out.fn_ext = sms ? pick<true, true>(lanes_c(N)) : pick<false, true>(lanes_c(N));
     out.smem = kMagicBytes + (size_t)kWarpsPerBlock * (L.bytes + (sms ? slot_bytes : 0u) + hash_bytes_for(N));
-    int dev = 0, sms_count = 0, per_sm = 0;
+    int dev = 0, sms_count = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms_count, cudaDevAttrMultiProcessorCount, dev);
-    if (e == cudaSuccess && out.smem > 48 * 1024)
-        e = cudaFuncSetAttribute(out.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)out.smem);
-    if (e == cudaSuccess)
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, out.fn, 32 * kWarpsPerBlock, out.smem);
-    if (e != cudaSuccess) return e;
-    if (per_sm < 1) return cudaErrorInvalidConfiguration;
     const long long want = ((long long)R + kWarpsPerBlock - 1) / kWarpsPerBlock;
-    out.grid = (int)std::min<long long>(want, (long long)sms_count * per_sm);
-    return cudaSuccess;
+    for (int v = 0; v < 2 && e == cudaSuccess; ++v) {
+        RunKernel fn = v ? out.fn_ext : out.fn;
+        int per_sm = 0;
+        if (out.smem > 48 * 1024)
+            e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)out.smem);
+        if (e == cudaSuccess)
+            e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, 32 * kWarpsPerBlock, out.smem);
+        if (e != cudaSuccess) return e;
+        if (per_sm < 1) return cudaErrorInvalidConfiguration;
+        (v ? out.grid_ext : out.grid) = (int)std::min<long long>(want, (long long)sms_count * per_sm);
+    }
+    return e;
 }
 
 inline unsigned long long magic40(unsigned d) { return ((1ull << kMagicShift) + d - 1ull) / d; }
@@ -1343,6 +1437,7 @@ struct sim {
     uint8_t *d_tier = nullptr;
     uint4 *d_node = nullptr;
     sim_request_result_t *d_res = nullptr;
+    uint32_t *d_drain = nullptr;  // [R][N] drain start times (sim_set_drain), or NULL
     int sms = 0;
     std::string err;
 };
@@ -1416,6 +1511,19 @@ void fill_scalars(mt::Params &p, const sim_cluster_t &cl, const sim_policy_t &po
     p.base = (int)pol.iter_base_us;
     p.a = (int)pol.iter_us_per_prefill_token;
     p.b = (int)pol.iter_us_per_decode_seq;
+    p.ticks = pol.enable_migration || pol.autoscale;
+    p.autoscale = pol.autoscale;
+    p.scale_out_num = pol.scale_out_num;
+    p.scale_in_num = pol.scale_in_num;
+    p.scale_den = pol.scale_den;
+    unsigned __int128 l = 1;  // lcm(1, ..., Bmax): every max(B, 1) divides it
+    for (unsigned d = 2; d <= (unsigned)cl.max_batch; ++d) {
+        unsigned a = d, b = (unsigned)(l % d);
+        while (b) { const unsigned t = a % b; a = b; b = t; }
+        l = l / a * d;
+    }
+    p.lcm_lo = (unsigned long long)l;
+    p.lcm_hi = (unsigned long long)(l >> 64);
     p.L = L;
     p.hash_bytes = mt::hash_bytes_for(cl.num_instances);
 }
@@ -1425,6 +1533,8 @@ mt::Params make_params(const sim_t *s, long long max_steps) {
     memset(&p, 0, sizeof p);
     fill_scalars(p, s->cl, s->pol, s->K, s->pol.event_log_capacity, s->L, max_steps);
     p.offsets = s->d_off;
+    p.drain_src = s->d_drain;
+    p.drains = s->d_drain != nullptr;
     p.arrival = s->d_arrival;
     p.plen = s->d_plen;
     p.olen = s->d_olen;
@@ -1505,6 +1615,12 @@ int validate_config(sim_t *s, const sim_cluster_t *cl, const sim_tier_table_t *t
         return fail(s, SIM_ERR_ARG, "event_log_capacity must be in [0, 2^24]");
     if (pol->migrate_interval_us < 1 || pol->migrate_interval_us > (1LL << 31))
         return fail(s, SIM_ERR_ARG, "migrate_interval_us must be in [1, 2^31]");
+    if (pol->autoscale != 0 && pol->autoscale != 1) return fail(s, SIM_ERR_ARG, "autoscale must be 0 or 1");
+    if (pol->autoscale && (pol->scale_den < 1 || pol->scale_den > 64 || pol->scale_out_num < -4096 ||
+                           pol->scale_in_num > 4096 || pol->scale_out_num >= pol->scale_in_num))
+        return fail(s, SIM_ERR_ARG,
+                    "auto-scaling thresholds must be num/den with den in [1, 64], numerators in [-4096, 4096] "
+                    "and scale_out_num < scale_in_num");
     return SIM_OK;
 }
 
@@ -1669,6 +1785,26 @@ int sim_reset(sim_t *s) {
     return reset_state(s);
 }
 
+int sim_set_drain(sim_t *s, const uint32_t *drain_start_us, int on_device) {
+    if (!s) return SIM_ERR_ARG;
+    if (on_device != 0 && on_device != 1) return fail(s, SIM_ERR_ARG, "on_device must be 0 or 1");
+    if (!drain_start_us) {
+        dfree(s, s->d_drain);
+        s->d_drain = nullptr;
+        return SIM_OK;
+    }
+    const size_t bytes = (size_t)s->cl.num_replicas * (size_t)s->cl.num_instances * 4u;
+    if (!s->d_drain) {
+        s->d_drain = (uint32_t *)dalloc(s, bytes);
+        if (!s->d_drain) return fail(s, SIM_ERR_OOM, "device allocation of the drain schedule failed");
+    }
+    cudaError_t e = cudaMemcpyAsync(s->d_drain, drain_start_us, bytes,
+                                    on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice, s->stream);
+    if (e == cudaSuccess && !on_device) e = cudaStreamSynchronize(s->stream);  // the host buffer may be reused
+    if (e != cudaSuccess) return cuda_fail(s, e, "sim_set_drain copy");
+    return SIM_OK;
+}
+
 int sim_run(sim_t *s, int64_t max_steps, int64_t *num_unfinished) {
     if (!s) return SIM_ERR_ARG;
     if (!s->loaded) return fail(s, SIM_ERR_STATE, "sim_run before sim_load_trace");
@@ -1676,7 +1812,10 @@ int sim_run(sim_t *s, int64_t max_steps, int64_t *num_unfinished) {
     cudaError_t e = cudaMemsetAsync(s->d_work, 0, 4, s->stream);
     if (e != cudaSuccess) return cuda_fail(s, e, "sim_run");
     mt::Params p = make_params(s, (long long)max_steps);
-    s->launch.fn<<<s->launch.grid, 32 * mt::kWarpsPerBlock, s->launch.smem, s->stream>>>(p);
+    if (p.drains || p.autoscale)
+        s->launch.fn_ext<<<s->launch.grid_ext, 32 * mt::kWarpsPerBlock, s->launch.smem, s->stream>>>(p);
+    else
+        s->launch.fn<<<s->launch.grid, 32 * mt::kWarpsPerBlock, s->launch.smem, s->stream>>>(p);
     int rc = check_launch(s, "k_run");
     if (rc) return rc;
     if (num_unfinished) {
@@ -1861,7 +2000,10 @@ extern "C" int sim_run_static(const sim_cluster_t *cl, const sim_tier_table_t *t
         const long long nb = std::min<long long>((n + 255) / 256, 65535LL * 16);
         mt::k_init_requests<<<(unsigned)nb, 256, 0, st>>>(per_request, (long long)n);
     }
-    lc.fn<<<lc.grid, 32 * mt::kWarpsPerBlock, lc.smem, st>>>(p);
+    if (p.autoscale)
+        lc.fn_ext<<<lc.grid_ext, 32 * mt::kWarpsPerBlock, lc.smem, st>>>(p);
+    else
+        lc.fn<<<lc.grid, 32 * mt::kWarpsPerBlock, lc.smem, st>>>(p);
     mt::k_export_stats<<<(R + 255) / 256, 256, 0, st>>>(p.rep, per_replica, R, nullptr);
     e = cudaGetLastError();
     if (e == cudaSuccess) e = cudaStreamSynchronize(st);

@@ -21,7 +21,7 @@ SIM_OK = 0
 SIM_ERR_ARG, SIM_ERR_TRACE, SIM_ERR_STATE, SIM_ERR_OOM = -1, -2, -3, -4
 SIM_ERR_OVERFLOW, SIM_ERR_CUDA, SIM_ERR_INTERNAL, SIM_ERR_DEADLOCK = -5, -7, -8, -10
 SIM_REPLICA_DONE, SIM_REPLICA_RUNNING = 0, 1
-SIM_EV_QUEUED, SIM_EV_START, SIM_EV_COMMIT, SIM_EV_ABORT = 0, 1, 2, 3
+SIM_EV_QUEUED, SIM_EV_START, SIM_EV_COMMIT, SIM_EV_ABORT, SIM_EV_SCALE_OUT, SIM_EV_SCALE_IN = 0, 1, 2, 3, 4, 5
 SIM_NONE32, SIM_NONE16 = 0xFFFFFFFF, 0xFFFF
 SIM_MAX_TIERS = 16
 
@@ -30,10 +30,11 @@ RESULT_DTYPE = np.dtype([("dispatch_instance", "<u2"), ("final_instance", "<u2")
 STATS_DTYPE = np.dtype([("steps", "<u8"), ("iterations", "<u8"), ("member_iterations", "<u8"), ("events", "<u8"),
                         ("migrations", "<u4"), ("preemptions", "<u4"), ("migration_starts", "<u4"),
                         ("migration_aborts", "<u4"), ("log_events", "<u4"), ("finished", "<u4"),
-                        ("last_time_us", "<u4"), ("status", "<i4")])
+                        ("last_time_us", "<u4"), ("status", "<i4"), ("scale_out_signals", "<u4"),
+                        ("scale_in_signals", "<u4")])
 EVENT_DTYPE = np.dtype([("time_us", "<u4"), ("request", "<u4"), ("blocks", "<u2"), ("src", "u1"), ("dst", "u1"),
                         ("kind", "u1"), ("pad", "u1", (3,))])
-assert RESULT_DTYPE.itemsize == 16 and STATS_DTYPE.itemsize == 64 and EVENT_DTYPE.itemsize == 16
+assert RESULT_DTYPE.itemsize == 16 and STATS_DTYPE.itemsize == 72 and EVENT_DTYPE.itemsize == 16
 
 
 class sim_cluster_t(ctypes.Structure):
@@ -53,7 +54,9 @@ class sim_policy_t(ctypes.Structure):
                 ("iter_base_us", ctypes.c_int64), ("iter_us_per_prefill_token", ctypes.c_int64),
                 ("iter_us_per_decode_seq", ctypes.c_int64), ("migrate_blocks_per_iter", ctypes.c_int32),
                 ("theta_num", ctypes.c_int32), ("theta_den", ctypes.c_int32),
-                ("event_log_capacity", ctypes.c_int32), ("migrate_interval_us", ctypes.c_int64)]
+                ("event_log_capacity", ctypes.c_int32), ("migrate_interval_us", ctypes.c_int64),
+                ("autoscale", ctypes.c_int32), ("scale_out_num", ctypes.c_int32), ("scale_in_num", ctypes.c_int32),
+                ("scale_den", ctypes.c_int32)]
 
 
 ALLOC_FN = ctypes.CFUNCTYPE(ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p)
@@ -65,7 +68,7 @@ class sim_allocator_t(ctypes.Structure):
 
 
 EXPORTS = ["sim_create", "sim_load_trace", "sim_reset", "sim_run", "sim_metrics", "sim_destroy",
-           "sim_last_error", "sim_strerror", "sim_device_bytes", "sim_run_static"]
+           "sim_last_error", "sim_strerror", "sim_device_bytes", "sim_run_static", "sim_set_drain"]
 SIM_STATIC_SCRATCH_BYTES = 32 << 20
 
 _LIB = None
@@ -89,6 +92,8 @@ def lib() -> ctypes.CDLL:
         L.sim_load_trace.restype = ctypes.c_int
         L.sim_reset.argtypes = [vp]
         L.sim_reset.restype = ctypes.c_int
+        L.sim_set_drain.argtypes = [vp, vp, ctypes.c_int]
+        L.sim_set_drain.restype = ctypes.c_int
         L.sim_run.argtypes = [vp, i64, ctypes.POINTER(i64)]
         L.sim_run.restype = ctypes.c_int
         L.sim_metrics.argtypes = [vp, vp, vp, vp, ctypes.c_int]
@@ -147,6 +152,10 @@ def sim_load_trace(handle, replica_offsets_ptr: int, arrival_ptr: int, prompt_pt
 
 def sim_reset(handle) -> int:
     return _check(lib().sim_reset(handle), handle)
+
+
+def sim_set_drain(handle, drain_ptr, on_device: int) -> int:
+    return _check(lib().sim_set_drain(handle, drain_ptr, on_device), handle)
 
 
 def sim_run(handle, max_steps_per_replica: int, want_unfinished: bool = True):
@@ -228,7 +237,9 @@ class Simulator:
                                     self._rt.ctypes.data)
         self._pol = sim_policy_t(0, w.enable_migration, w.iter_base_us, w.iter_us_per_prefill_token,
                                  w.iter_us_per_decode_seq, w.migrate_blocks_per_iter, w.theta_num, w.theta_den,
-                                 self.event_log_capacity, w.migrate_interval_us)
+                                 self.event_log_capacity, w.migrate_interval_us, getattr(w, "autoscale", 0),
+                                 getattr(w, "scale_out_num", -1), getattr(w, "scale_in_num", 3),
+                                 getattr(w, "scale_den", 2))
         self._alloc = TorchAllocator(self.device) if torch_allocator else None
         self.handle = sim_create(self._cl, self._tt, self._pol, self.stream.cuda_stream,
                                  self._alloc.struct if self._alloc else None)
@@ -247,6 +258,12 @@ class Simulator:
     def load(self, on_device: bool = True) -> None:
         w = self.w
         self._off = np.ascontiguousarray(w.offsets, np.int64)
+        drain = getattr(w, "drain_start_us", None)
+        if drain is not None:
+            d = np.ascontiguousarray(drain, np.uint32)
+            if d.shape != (w.num_replicas, w.num_instances):
+                raise ValueError("drain_start_us must be [num_replicas, num_instances]")
+            sim_set_drain(self.handle, d.ctypes.data, 0)
         if on_device:
             tr = self._trace or self.device_trace()
             ptrs = [x.data_ptr() for x in tr]

@@ -6,7 +6,8 @@ from oracle import oracle as O
 from paper_2608_16336_gb300 import mtsim
 
 STAT_FIELDS = ("steps", "iterations", "member_iterations", "events", "migrations", "preemptions",
-               "migration_starts", "migration_aborts", "log_events", "finished")
+               "migration_starts", "migration_aborts", "log_events", "finished", "scale_out_signals",
+               "scale_in_signals")
 
 
 def run_gpu(w, *, event_log_capacity=4096, max_steps=None, on_device=True, torch_allocator=True):

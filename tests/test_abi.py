@@ -38,9 +38,9 @@ def test_library_exports_every_declared_symbol(L):
 
 def test_struct_sizes_match_header():
     assert ctypes.sizeof(mtsim.sim_cluster_t) == 20
-    assert ctypes.sizeof(mtsim.sim_policy_t) == 56
+    assert ctypes.sizeof(mtsim.sim_policy_t) == 72
     assert mtsim.RESULT_DTYPE.itemsize == 16
-    assert mtsim.STATS_DTYPE.itemsize == 64
+    assert mtsim.STATS_DTYPE.itemsize == 72
     assert mtsim.EVENT_DTYPE.itemsize == 16
 
 
@@ -77,6 +77,22 @@ def test_create_rejects_bad_policy(L, field, value):
     out = ctypes.c_void_p()
     rc = L.sim_create(ctypes.byref(cl), ctypes.byref(tt), ctypes.byref(pol), None, None, ctypes.byref(out))
     assert rc == mtsim.SIM_ERR_ARG
+
+
+@pytest.mark.parametrize("fields", [
+    dict(autoscale=2), dict(autoscale=1, scale_out_num=-1, scale_in_num=3, scale_den=0),
+    dict(autoscale=1, scale_out_num=-1, scale_in_num=3, scale_den=65),
+    dict(autoscale=1, scale_out_num=3, scale_in_num=3, scale_den=2),
+    dict(autoscale=1, scale_out_num=-5000, scale_in_num=3, scale_den=2),
+    dict(autoscale=1, scale_out_num=-1, scale_in_num=4097, scale_den=2)])
+def test_create_rejects_bad_autoscale(L, fields):
+    cl, tt, pol, keep = _valid()
+    for k, v in fields.items():
+        setattr(pol, k, v)
+    out = ctypes.c_void_p()
+    rc = L.sim_create(ctypes.byref(cl), ctypes.byref(tt), ctypes.byref(pol), None, None, ctypes.byref(out))
+    assert rc == mtsim.SIM_ERR_ARG and not out.value
+    assert b"auto" in L.sim_last_error(None)
 
 
 def test_create_rejects_bad_tier_tables(L):
@@ -116,6 +132,7 @@ def test_allocation_failure_is_reported(L):
 def test_null_object_calls(L):
     assert L.sim_run(None, 10, None) == mtsim.SIM_ERR_ARG
     assert L.sim_reset(None) == mtsim.SIM_ERR_ARG
+    assert L.sim_set_drain(None, None, 0) == mtsim.SIM_ERR_ARG
     assert L.sim_metrics(None, None, None, None, 0) == mtsim.SIM_ERR_ARG
     assert L.sim_load_trace(None, None, None, None, None, None, 0) == mtsim.SIM_ERR_ARG
     assert L.sim_device_bytes(None) == 0

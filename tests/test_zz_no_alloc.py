@@ -42,9 +42,9 @@ def _static_run(torch, w, cap):
     dev = torch.device("cuda", 0)
     tr = [torch.from_numpy(np.ascontiguousarray(a)).to(dev) for a in
           (w.arrival_us.view(np.int32), w.prompt_len.view(np.int16), w.output_len.view(np.int16), w.tier)]
-    res = torch.empty(w.total_requests * 16, dtype=torch.uint8, device=dev)
-    st = torch.empty(R * 64, dtype=torch.uint8, device=dev)
-    ev = torch.empty(R * cap * 16, dtype=torch.uint8, device=dev)
+    res = torch.empty(w.total_requests * mtsim.RESULT_DTYPE.itemsize, dtype=torch.uint8, device=dev)
+    st = torch.empty(R * mtsim.STATS_DTYPE.itemsize, dtype=torch.uint8, device=dev)
+    ev = torch.empty(R * cap * mtsim.EVENT_DTYPE.itemsize, dtype=torch.uint8, device=dev)
     torch.cuda.synchronize()
     mtsim.sim_run_static(cl, tt, pol, off.ctypes.data, *[x.data_ptr() for x in tr], res.data_ptr(), st.data_ptr(),
                          ev.data_ptr(), torch.cuda.current_stream().cuda_stream)
