@@ -204,6 +204,7 @@ def bench_gpu(args):
 
     res, st, _ = sim.metrics()
     assert (st["status"] == mtsim.SIM_REPLICA_DONE).all(), "a replica did not finish"
+    lat_info = time_latency_stats(torch, mtsim, sim, w, stream)
     steps_per_run = float(st["steps"].sum())
     events_per_run = float(st["events"].sum())
     member_iters = float(st["member_iterations"].sum())
@@ -280,6 +281,7 @@ def bench_gpu(args):
             "algorithmic_bytes_per_launch": alg_bytes,
         },
         "clocks": clk,
+        "aux_kernels": [lat_info],
     }
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(w, args.cpu_replicas)
@@ -289,6 +291,32 @@ def bench_gpu(args):
         import torch.distributed as dist
 
         dist.destroy_process_group()
+
+
+def time_latency_stats(torch, mtsim, sim, w, stream, reps: int = 10) -> dict:
+    """CUDA-event time of the per-tier latency reduction (sim_latency_stats) over the
+    finished simulation, device output, outside the timed step.  Its inputs
+    (16 + 4 + 2 + 1 bytes per request) are larger than L2 at this size."""
+    R, Q = w.num_replicas, w.total_requests
+    kmax = max(w.tables_k)
+    out = torch.empty(R * kmax * 3 * mtsim.LATENCY_DTYPE.itemsize, dtype=torch.uint8, device=stream.device)
+    for _ in range(3):
+        mtsim.sim_latency_stats(sim.handle, out.data_ptr(), 1)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
+    torch.cuda.synchronize()
+    for a, b in ev:
+        a.record(stream)
+        mtsim.sim_latency_stats(sim.handle, out.data_ptr(), 1)
+        b.record(stream)
+    torch.cuda.synchronize()
+    ms = sum(a.elapsed_time(b) for a, b in ev) / reps
+    nbytes = Q * (16 + 4 + 2 + 1) + out.numel()
+    peak, kind = measured_peak_hbm()
+    gbs = nbytes / (ms / 1e3) / 1e9
+    return {"kernel": "k_latency_hist + k_latency_pct (sim_latency_stats, output clear included)",
+            "work": "per-tier TTFT/TBT/E2E histograms and percentiles of every request",
+            "bound": "hbm", "ms": ms, "algorithmic_bytes_per_launch": nbytes, "achieved": gbs, "peak": peak,
+            "peak_kind": kind, "unit": "GB/s", "frac": gbs / peak}
 
 
 def cpu_baseline(w, nrep: int) -> dict:

@@ -173,6 +173,28 @@ typedef struct {
     uint8_t pad[3];
 } sim_migration_event_t;
 
+/* Per-tier latency statistics of one measure (Sec. 5.1, Sec. 5.3: the paper
+ * reports TTFT, time between tokens and end-to-end latency per priority tier,
+ * as distributions, means and P50 / P90 / P99).  992 bytes. */
+#define SIM_HIST_BUCKETS 240
+#define SIM_LAT_TTFT 0  /* first_token - arrival (prefill latency) */
+#define SIM_LAT_TBT 1   /* floor((finish - first_token) / (O - 1)), requests with O >= 2 */
+#define SIM_LAT_E2E 2   /* finish - arrival */
+typedef struct {
+    uint32_t count;              /* finished requests of the tier counted */
+    uint32_t max_us;             /* exact maximum (0 if count = 0) */
+    uint64_t sum_us;             /* exact sum; mean = sum_us / count */
+    uint32_t p50_us, p90_us, p99_us; /* nearest-rank percentiles (the value of rank ceil(p * count / 100)),
+                                        rounded down to the floor of their histogram bucket: within
+                                        1/8 below the exact value; 0 if count = 0 */
+    uint32_t pad;
+    /* hist[b]: requests whose value v falls in bucket b: b = v for v < 8,
+     * else b = 8 * (e - 3) + floor(v / 2^(e-3)) with e = floor(log2 v):
+     * eight equal buckets per power of two, floors 0..7, 8, 9, .., 15, 16,
+     * 18, .., 30, 32, 36, ... */
+    uint32_t hist[SIM_HIST_BUCKETS];
+} sim_latency_stats_t;
+
 /* Optional device allocator, e.g. a framework's caching allocator.  alloc
  * returns a device pointer (16-byte aligned at least) or NULL; free releases
  * one.  Both are called on the calling host thread with the simulation's
@@ -245,6 +267,16 @@ int sim_run(sim_t *sim, int64_t max_steps_per_replica, int64_t *num_unfinished);
  * simulation produced them. */
 int sim_metrics(sim_t *sim, sim_request_result_t *per_request, sim_replica_stats_t *per_replica,
                 sim_migration_event_t *events, int on_device);
+
+/* Per-tier latency statistics of the current results, computed on the device:
+ * out[(r * max_tiers + k) * 3 + m] for replica r, tier k < max_tiers (tiers
+ * beyond a replica's K have count 0) and measure m = SIM_LAT_*.  Counts only
+ * requests that have finished, so it may be called between sim_run calls.
+ * out is host or device per on_device, [R * max_tiers * 3] records.  Host
+ * output synchronises the stream (and allocates a device staging buffer of
+ * the same size on first use); device output is asynchronous.  Returns
+ * SIM_ERR_STATE before sim_load_trace. */
+int sim_latency_stats(sim_t *sim, sim_latency_stats_t *out, int on_device);
 
 /* Releases everything the object owns (synchronises the stream first).
  * NULL is ignored. */

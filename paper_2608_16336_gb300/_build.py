@@ -60,16 +60,23 @@ def mtsim_sources() -> list[str]:
 
 
 def build_mtsim(force: bool = False, extra_flags: list[str] | None = None) -> str:
+    """Compiles every csrc/*.cu to an object in parallel, then links libmtsim.so."""
     srcs = mtsim_sources()
     if force or extra_flags or _stale(MTSIM_SO, srcs):
-        os.makedirs(LIB_DIR, exist_ok=True)
+        obj_dir = os.path.join(LIB_DIR, "obj")
+        os.makedirs(obj_dir, exist_ok=True)
+        cus = [s for s in srcs if s.endswith(".cu")]
+        tag = "%d" % os.getpid()
+        objs = [os.path.join(obj_dir, os.path.basename(c)[:-3] + ".%s.o" % tag) for c in cus]
+        flags = [ARCH, "-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I", INCLUDE] + list(extra_flags or [])
+        with ThreadPoolExecutor(len(cus)) as ex:
+            for f in [ex.submit(_run, [_nvcc(), "-c", c, "-o", o] + flags) for c, o in zip(cus, objs)]:
+                f.result()
         tmp = MTSIM_SO + ".tmp%d" % os.getpid()
-        cmd = [
-            _nvcc(), ARCH, "-O3", "-lineinfo", "-std=c++17", "-shared", "-Xcompiler", "-fPIC",
-            "-I", INCLUDE, os.path.join(CSRC, "mtsim.cu"), "-o", tmp,
-        ] + list(extra_flags or [])
-        _run(cmd)
+        _run([_nvcc(), ARCH, "-shared", "-Xcompiler", "-fPIC", *objs, "-o", tmp])
         os.replace(tmp, MTSIM_SO)
+        for o in objs:
+            os.remove(o)
     return MTSIM_SO
 
 

@@ -46,6 +46,7 @@
 //   an inconsistency into SIM_ERR_INTERNAL for that replica instead of an
 //   out-of-bounds access.
 #include "mtsim.h"
+#include "latency.cuh"
 
 #include <cuda_runtime.h>
 
@@ -1438,6 +1439,10 @@ struct sim {
     uint4 *d_node = nullptr;
     sim_request_result_t *d_res = nullptr;
     uint32_t *d_drain = nullptr;  // [R][N] drain start times (sim_set_drain), or NULL
+    sim_latency_stats_t *d_lat = nullptr;  // device staging of sim_latency_stats for host output
+    int *d_lat_rep = nullptr;              // chunk table of sim_latency_stats: replica and first record
+    long long *d_lat_b0 = nullptr;
+    int lat_nchunks = -1;                  // -1: to be built for the loaded trace
     int sms = 0;
     std::string err;
 };
@@ -1743,6 +1748,7 @@ int sim_load_trace(sim_t *s, const int64_t *off, const uint32_t *arrival, const 
         if (!s->d_off) return fail(s, SIM_ERR_OOM, "device allocation failed");
     }
     s->h_off.assign(off, off + R + 1);
+    s->lat_nchunks = -1;
     const cudaMemcpyKind kind = on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
     cudaError_t e = cudaMemcpyAsync(s->d_off, s->h_off.data(), ((size_t)R + 1) * 8, cudaMemcpyHostToDevice, s->stream);
     if (n > 0) {
@@ -1783,6 +1789,59 @@ int sim_reset(sim_t *s) {
     if (!s) return SIM_ERR_ARG;
     if (!s->loaded) return fail(s, SIM_ERR_STATE, "sim_reset before sim_load_trace");
     return reset_state(s);
+}
+
+static_assert(sizeof(sim_latency_stats_t) == 32 + 4 * SIM_HIST_BUCKETS, "sim_latency_stats_t layout");
+
+int sim_latency_stats(sim_t *s, sim_latency_stats_t *out, int on_device) {
+    if (!s) return SIM_ERR_ARG;
+    if (!out) return fail(s, SIM_ERR_ARG, "out is NULL");
+    if (on_device != 0 && on_device != 1) return fail(s, SIM_ERR_ARG, "on_device must be 0 or 1");
+    if (!s->loaded) return fail(s, SIM_ERR_STATE, "sim_latency_stats before sim_load_trace");
+    const int R = s->cl.num_replicas, KT = s->K;
+    const size_t n = (size_t)R * KT * 3;
+    sim_latency_stats_t *d = out;
+    if (!on_device) {
+        if (!s->d_lat) {
+            s->d_lat = (sim_latency_stats_t *)dalloc(s, n * sizeof(sim_latency_stats_t));
+            if (!s->d_lat) return fail(s, SIM_ERR_OOM, "device allocation of the latency statistics failed");
+        }
+        d = s->d_lat;
+    }
+    if (s->lat_nchunks < 0) {  // chunk table of the loaded trace
+        std::vector<int> rep;
+        std::vector<long long> b0;
+        for (int r = 0; r < R; ++r)
+            for (long long b = s->h_off[r]; b < s->h_off[r + 1]; b += mtlat::kChunk) {
+                rep.push_back(r);
+                b0.push_back(b);
+            }
+        const int nc = (int)rep.size();
+        dfree(s, s->d_lat_rep);
+        dfree(s, s->d_lat_b0);
+        s->d_lat_rep = nullptr;
+        s->d_lat_b0 = nullptr;
+        if (nc > 0) {
+            s->d_lat_rep = (int *)dalloc(s, (size_t)nc * 4);
+            s->d_lat_b0 = (long long *)dalloc(s, (size_t)nc * 8);
+            if (!s->d_lat_rep || !s->d_lat_b0) return fail(s, SIM_ERR_OOM, "device allocation of the chunk table failed");
+            cudaError_t e = cudaMemcpyAsync(s->d_lat_rep, rep.data(), (size_t)nc * 4, cudaMemcpyHostToDevice, s->stream);
+            if (e == cudaSuccess)
+                e = cudaMemcpyAsync(s->d_lat_b0, b0.data(), (size_t)nc * 8, cudaMemcpyHostToDevice, s->stream);
+            if (e == cudaSuccess) e = cudaStreamSynchronize(s->stream);  // the host vectors go out of scope
+            if (e != cudaSuccess) return cuda_fail(s, e, "sim_latency_stats chunk table");
+        }
+        s->lat_nchunks = nc;
+    }
+    cudaError_t e = mtlat::launch(s->d_lat_rep, s->d_lat_b0, s->lat_nchunks, s->d_off, KT, s->d_arrival, s->d_olen,
+                                  s->d_tier, s->d_res, d, (long long)n, s->sms, s->stream);
+    if (e != cudaSuccess) return cuda_fail(s, e, "sim_latency_stats");
+    if (!on_device) {
+        e = cudaMemcpyAsync(out, d, n * sizeof(sim_latency_stats_t), cudaMemcpyDeviceToHost, s->stream);
+        if (e == cudaSuccess) e = cudaStreamSynchronize(s->stream);
+        if (e != cudaSuccess) return cuda_fail(s, e, "sim_latency_stats copy");
+    }
+    return SIM_OK;
 }
 
 int sim_set_drain(sim_t *s, const uint32_t *drain_start_us, int on_device) {

@@ -34,7 +34,12 @@ STATS_DTYPE = np.dtype([("steps", "<u8"), ("iterations", "<u8"), ("member_iterat
                         ("scale_in_signals", "<u4")])
 EVENT_DTYPE = np.dtype([("time_us", "<u4"), ("request", "<u4"), ("blocks", "<u2"), ("src", "u1"), ("dst", "u1"),
                         ("kind", "u1"), ("pad", "u1", (3,))])
+SIM_HIST_BUCKETS = 240
+SIM_LAT_TTFT, SIM_LAT_TBT, SIM_LAT_E2E = 0, 1, 2
+LATENCY_DTYPE = np.dtype([("count", "<u4"), ("max_us", "<u4"), ("sum_us", "<u8"), ("p50_us", "<u4"),
+                          ("p90_us", "<u4"), ("p99_us", "<u4"), ("pad", "<u4"), ("hist", "<u4", (SIM_HIST_BUCKETS,))])
 assert RESULT_DTYPE.itemsize == 16 and STATS_DTYPE.itemsize == 72 and EVENT_DTYPE.itemsize == 16
+assert LATENCY_DTYPE.itemsize == 992
 
 
 class sim_cluster_t(ctypes.Structure):
@@ -68,7 +73,8 @@ class sim_allocator_t(ctypes.Structure):
 
 
 EXPORTS = ["sim_create", "sim_load_trace", "sim_reset", "sim_run", "sim_metrics", "sim_destroy",
-           "sim_last_error", "sim_strerror", "sim_device_bytes", "sim_run_static", "sim_set_drain"]
+           "sim_last_error", "sim_strerror", "sim_device_bytes", "sim_run_static", "sim_set_drain",
+           "sim_latency_stats"]
 SIM_STATIC_SCRATCH_BYTES = 32 << 20
 
 _LIB = None
@@ -94,6 +100,8 @@ def lib() -> ctypes.CDLL:
         L.sim_reset.restype = ctypes.c_int
         L.sim_set_drain.argtypes = [vp, vp, ctypes.c_int]
         L.sim_set_drain.restype = ctypes.c_int
+        L.sim_latency_stats.argtypes = [vp, vp, ctypes.c_int]
+        L.sim_latency_stats.restype = ctypes.c_int
         L.sim_run.argtypes = [vp, i64, ctypes.POINTER(i64)]
         L.sim_run.restype = ctypes.c_int
         L.sim_metrics.argtypes = [vp, vp, vp, vp, ctypes.c_int]
@@ -156,6 +164,10 @@ def sim_reset(handle) -> int:
 
 def sim_set_drain(handle, drain_ptr, on_device: int) -> int:
     return _check(lib().sim_set_drain(handle, drain_ptr, on_device), handle)
+
+
+def sim_latency_stats(handle, out_ptr, on_device: int) -> int:
+    return _check(lib().sim_latency_stats(handle, out_ptr, on_device), handle)
 
 
 def sim_run(handle, max_steps_per_replica: int, want_unfinished: bool = True):
@@ -288,6 +300,13 @@ class Simulator:
         sim_metrics(self.handle, res.ctypes.data if len(res) else None, st.ctypes.data,
                     ev.ctypes.data if self.event_log_capacity else None, 0)
         return res, st, ev.reshape(w.num_replicas, -1)[:, : self.event_log_capacity]
+
+    def latency_stats(self) -> np.ndarray:
+        """Per-tier TTFT / TBT / E2E statistics, LATENCY_DTYPE [R, max tiers, 3]."""
+        kmax = max(self.w.tables_k)
+        out = np.empty(self.w.num_replicas * kmax * 3, LATENCY_DTYPE)
+        sim_latency_stats(self.handle, out.ctypes.data, 0)
+        return out.reshape(self.w.num_replicas, kmax, 3)
 
     def events_of(self, ev, st, r: int) -> np.ndarray:
         """Replica r's migration log as an (n, 6) int64 array: time, request, src, dst, blocks, kind."""

@@ -42,6 +42,7 @@ def test_struct_sizes_match_header():
     assert mtsim.RESULT_DTYPE.itemsize == 16
     assert mtsim.STATS_DTYPE.itemsize == 72
     assert mtsim.EVENT_DTYPE.itemsize == 16
+    assert mtsim.LATENCY_DTYPE.itemsize == 992
 
 
 def _valid():
@@ -133,6 +134,7 @@ def test_null_object_calls(L):
     assert L.sim_run(None, 10, None) == mtsim.SIM_ERR_ARG
     assert L.sim_reset(None) == mtsim.SIM_ERR_ARG
     assert L.sim_set_drain(None, None, 0) == mtsim.SIM_ERR_ARG
+    assert L.sim_latency_stats(None, None, 0) == mtsim.SIM_ERR_ARG
     assert L.sim_metrics(None, None, None, None, 0) == mtsim.SIM_ERR_ARG
     assert L.sim_load_trace(None, None, None, None, None, None, 0) == mtsim.SIM_ERR_ARG
     assert L.sim_device_bytes(None) == 0

@@ -1,0 +1,125 @@
+"""Per-tier latency statistics on the GPU (sim_latency_stats) vs the oracle's
+statistics of the oracle's own results, bit-exact: counts, sums, maxima,
+every histogram bucket and the P50 / P90 / P99 floors."""
+import numpy as np
+import pytest
+
+from oracle import latency as LT
+from oracle import oracle as O
+from paper_2608_16336_gb300 import mtsim
+from paper_2608_16336_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    torch.cuda.set_device(0)
+
+
+def gpu_stats(w, max_steps=None):
+    sim = mtsim.Simulator(w, event_log_capacity=0)
+    try:
+        sim.load()
+        sim.run() if max_steps is None else sim.run(max_steps)
+        return sim.latency_stats()
+    finally:
+        sim.close()
+
+
+def compare(w, got, replicas, max_steps=1 << 62):
+    kmax = max(w.tables_k)
+    ref = O.run_workload(w, replicas, nthreads=8, log_capacity=0, max_steps=max_steps)
+    for r in replicas:
+        sl = w.replica_slice(r)
+        want = LT.replica_stats(w.arrival_us[sl], w.output_len[sl], w.tier[sl], ref[r].first_token_us,
+                                ref[r].finish_us, kmax)
+        for k in range(kmax):
+            for m in range(3):
+                g, s = got[r, k, m], want[k][m]
+                where = (r, k, LT.METRICS[m])
+                assert int(g["count"]) == s["count"], where
+                assert int(g["sum_us"]) == s["sum"], where
+                assert int(g["max_us"]) == s["max"], where
+                assert [int(x) for x in g["hist"]] == s["hist"], where
+                assert (int(g["p50_us"]), int(g["p90_us"]), int(g["p99_us"])) == (s["p50"], s["p90"], s["p99"]), where
+
+
+def test_workload0():
+    w = W.config(0)
+    compare(w, gpu_stats(w), [0])
+
+
+def test_workload1_slice():
+    w = W.config(1, replicas=range(67), requests=3000)
+    compare(w, gpu_stats(w), range(67))
+
+
+def test_workload2_mixed_tier_counts():
+    reps = [((k * 3 + d) * 2 + ld) * 64 + (k + d) % 64 for k in range(10) for d in range(3) for ld in range(2)]
+    w = W.config(2, replicas=reps, requests=1500)
+    got = gpu_stats(w)
+    compare(w, got, range(w.num_replicas))
+    # tiers a replica does not have are empty
+    for r in range(w.num_replicas):
+        assert (got[r, w.replica_k(r):]["count"] == 0).all()
+
+
+def test_workload3_many_instances():
+    w = W.config(3, replicas=[0, 1], requests=20000)
+    compare(w, gpu_stats(w), [0, 1])
+
+
+def test_unfinished_requests_are_left_out():
+    w = W.config(1, replicas=range(6), requests=2000)
+    got = gpu_stats(w, max_steps=3000)
+    compare(w, got, range(6), max_steps=3000)
+    assert 0 < got[:, :, mtsim.SIM_LAT_E2E]["count"].sum() < w.total_requests
+
+
+def test_sixteen_tiers_and_empty_replicas():
+    rng = np.random.default_rng(5)
+    traces = []
+    for r in range(9):
+        q = 0 if r % 4 == 0 else int(rng.integers(1, 300))
+        a = np.sort(rng.integers(0, 200_000, size=q)).astype(np.uint32)
+        p = rng.integers(1, 600, size=q).astype(np.uint16)
+        o = rng.integers(1, 200, size=q).astype(np.uint16)
+        traces.append((a, p, o, rng.integers(0, 16, size=q).astype(np.uint8)))
+    h = [max(0, 256 >> i) for i in range(16)]
+    w = W.custom(8, 1024, [16], [h], [0] * 9, traces)
+    got = gpu_stats(w)
+    compare(w, got, range(9))
+    assert (got[0]["count"] == 0).all() and (got[0]["p99_us"] == 0).all()
+
+
+def test_device_output_equals_host_output():
+    torch = pytest.importorskip("torch")
+    w = W.config(1, replicas=range(5), requests=1000)
+    sim = mtsim.Simulator(w, event_log_capacity=0)
+    try:
+        sim.load()
+        sim.run()
+        host = sim.latency_stats()
+        d = torch.empty(host.size * mtsim.LATENCY_DTYPE.itemsize, dtype=torch.uint8, device="cuda")
+        mtsim.sim_latency_stats(sim.handle, d.data_ptr(), 1)
+        torch.cuda.synchronize()
+        dev = d.cpu().numpy().view(mtsim.LATENCY_DTYPE).reshape(host.shape)
+    finally:
+        sim.close()
+    assert host.tobytes() == dev.tobytes()
+
+
+def test_full_workload1_sampled_and_consistent():
+    w = W.config(1)
+    got = gpu_stats(w)
+    compare(w, got, [0, 400, 1023])
+    # every request finished once: TTFT and E2E counts add up to the trace
+    assert int(got[:, :, mtsim.SIM_LAT_TTFT]["count"].sum()) == w.total_requests
+    assert int(got[:, :, mtsim.SIM_LAT_E2E]["count"].sum()) == w.total_requests
+    # per-tier TTFT ordering under load (Sec. 5.1): tier 0 before tier 3 in the median
+    p50 = got[:, :, mtsim.SIM_LAT_TTFT]["p50_us"].astype(np.int64)
+    assert (p50[:, 0] <= p50[:, 3]).mean() > 0.9
