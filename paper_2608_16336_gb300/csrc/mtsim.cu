@@ -457,6 +457,40 @@ __device__ __forceinline__ void coop_finish(const Ctx &x, Cnt &cn, int i) {
     __syncwarp();
 }
 
+// Phase 1, second part, one lane: the requests of instance i whose output is
+// complete finish at x.t and free their KV, for an instance in no migration
+// (so nothing outside instance i changes).  The owner lane scans its slots
+// (independent loads) and compacts them in order.  Returns how many finished;
+// the caller adds them to the replica's count.
+__device__ __forceinline__ uint32_t solo_finish(const Ctx &x, Cnt &cn, int i) {
+    const int n = x.nrun[i];
+    const uint32_t nf = x.nf[i];
+    uint4 *p = slot_ptr(x, i, 0);
+    int w = 0, freed = 0;
+    uint32_t fm = kNone, nfin = 0;
+    for (int q = 0; q < n; ++q) {
+        const uint4 sl = p[q];
+        const uint32_t fin = sl_fin(sl);
+        if (fin == nf) {
+            x.res[sl.x].finish_us = x.t;
+            x.res[sl.x].final_instance = (uint16_t)i;
+            freed += blocks_for(x, sl_c(sl) + nf - sl.y);
+            cnt_dec(x, i, (int)sl_tier(sl));
+            x.hist[i * x.TH + sl_rho(sl)]--;
+            ++nfin;
+        } else {
+            if (w != q) p[w] = sl;
+            ++w;
+            fm = min(fm, fin);
+        }
+    }
+    x.free_[i] += freed;
+    x.nrun[i] = (uint8_t)w;
+    x.minfin[i] = fm;
+    cn.events += nfin;
+    return nfin;
+}
+
 // One copy stage at the end of an iteration of migration source s, whole
 // warp: up to S of the request's blocks are reserved on the destination
 // (abandoning the migration if they do not fit), and the request commits
@@ -1076,7 +1110,7 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
                 }
                 uint32_t fresh = 0;  // distinct event times this lane contributes (C > 1)
                 uint32_t tlast = 0;  // latest event time processed in the window
-                uint32_t pend = 0;   // instances whose finishing requests the warp handles next
+                uint32_t sfin = 0;   // requests this lane's instances finished in the window
 #pragma unroll
                 for (int j = 0; j < C; ++j) {
                     if (!((solo >> j) & 1u)) continue;
@@ -1084,27 +1118,10 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
                     x.t = bz[j];
                     tlast = max(tlast, bz[j]);
                     if (C > 1) fresh += tset_insert(x, bz[j]);
-                    if (inst_complete_head(x, i)) pend |= 1u << j;
-                    else inst_form(x, cn, i, p.base, p.a, p.b);
+                    if (inst_complete_head(x, i)) sfin += solo_finish(x, cn, i);
+                    inst_form(x, cn, i, p.base, p.a, p.b);
                 }
                 __syncwarp();
-                {
-                    uint32_t pl = __ballot_sync(kFull, pend != 0);
-                    while (pl) {
-                        const int l = __ffs(pl) - 1;
-                        pl &= pl - 1;
-                        uint32_t h = C == 1 ? 1u : __shfl_sync(kFull, pend, l);
-                        while (h) {
-                            const int j = __ffs(h) - 1;
-                            h &= h - 1;
-                            const int i = l * C + j;
-                            x.t = __shfl_sync(kFull, bz[j], l);
-                            coop_finish(x, cn, i);
-                            if (lane == 0) inst_form(x, cn, i, p.base, p.a, p.b);
-                            __syncwarp();
-                        }
-                    }
-                }
                 uint32_t ucount, u = kNone;
                 if (C == 1) {
                     u = solo ? bz[0] : kNone;
@@ -1145,7 +1162,8 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
                 }
                 cn.steps += ucount;
                 x.t = __reduce_max_sync(kFull, tlast);
-                cn.finished = __shfl_sync(kFull, cn.finished, 0);  // finishes are all counted on lane 0
+                // lane 0 counted the finishes of steps in time order; the lanes, their own
+                cn.finished = __shfl_sync(kFull, cn.finished, 0) + __reduce_add_sync(kFull, sfin);
                 const int ws = __reduce_min_sync(kFull, cn.status);
                 cn.status = ws;
                 if (cn.status < 0) break;
