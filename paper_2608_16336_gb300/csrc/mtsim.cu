@@ -345,15 +345,19 @@ __device__ __forceinline__ uint4 *slot_ptr(const Ctx &x, int i, int s) { return 
 
 // A request joins instance i's running list at position n with context c and
 // remaining output left; its first formation there will be number nf + 1.
-__device__ __forceinline__ void slot_join(const Ctx &x, int i, int n, uint32_t r, uint32_t c, uint32_t left,
-                                          uint32_t tier) {
-    const uint32_t phi = x.nf[i] + 1u;
-    const uint32_t pm = x.phase[i] + 1u == (uint32_t)x.T ? 0u : x.phase[i] + 1u;  // phi mod T
+__device__ __forceinline__ void slot_join_at(const Ctx &x, int i, int n, uint32_t r, uint32_t c, uint32_t left,
+                                             uint32_t tier, uint32_t nf, uint32_t ph) {
+    const uint32_t phi = nf + 1u;
+    const uint32_t pm = ph + 1u == (uint32_t)x.T ? 0u : ph + 1u;  // phi mod T
     const uint32_t cm = mod_t(x, c);
     const uint32_t rho = cm >= pm ? cm - pm : cm + (uint32_t)x.T - pm;
     *slot_ptr(x, i, n) = make_uint4(r, phi, c | (left << 16), tier | (rho << 16));
     x.hist[i * x.TH + rho]++;
     x.minfin[i] = min(x.minfin[i], phi + left - 1u);
+}
+__device__ __forceinline__ void slot_join(const Ctx &x, int i, int n, uint32_t r, uint32_t c, uint32_t left,
+                                          uint32_t tier) {
+    slot_join_at(x, i, n, r, c, left, tier, x.nf[i], x.phase[i]);
 }
 
 // Removes slot s of instance i's running list (order kept); returns its record.
@@ -551,13 +555,20 @@ __device__ __forceinline__ void preempt_book(const Ctx &x, Cnt &cn, int i, const
 // one when out of blocks; (ii) admission in (tier, FCFS) order while the head
 // of line fits; (iii) the iteration starts.
 __device__ __forceinline__ void inst_form(const Ctx &x, Cnt &cn, int i, int base, int a_us, int b_us) {
+    // the instance's scalars, read together up front (the code below would
+    // otherwise reload them after every shared-memory store)
     int n = x.nrun[i];
+    int fr = x.free_[i];
+    const uint32_t ph = x.phase[i];
+    const uint32_t nf = x.nf[i];
+    uint32_t wm = x.wmask[i];
+    int need = x.hol[i];
     if (n > 0) {
-        const uint32_t ph = x.phase[i];
         const int deficit = x.hist[i * x.TH + (ph == 0 ? 0u : (uint32_t)x.T - ph)];
-        if (deficit <= x.free_[i]) {
-            x.free_[i] -= deficit;  // every request that needs a block gets it
+        if (deficit <= fr) {
+            fr -= deficit;  // every request that needs a block gets it
         } else {
+            x.free_[i] = fr;
             // In running order, a request that needs a block (at most one)
             // takes a free one or preempts the lowest-priority newest running
             // request, possibly itself.  Positions are the list's before this
@@ -569,11 +580,11 @@ __device__ __forceinline__ void inst_form(const Ctx &x, Cnt &cn, int i, int base
                 const uint4 sl = p[q];
                 if (blocks_for(x, sl_c(sl) + sl_adv(x, i, sl)) > sl_blocks(x, i, sl)) needs |= 1ull << q;
             }
-            int fr = x.free_[i];
+            int fb = x.free_[i];
             for (int q = 0; q < n; ++q) {
                 if (!((alive & needs) >> q & 1ull)) continue;
                 for (;;) {
-                    if (fr > 0) { --fr; granted |= 1ull << q; break; }
+                    if (fb > 0) { --fb; granted |= 1ull << q; break; }
                     int v = -1;
                     uint32_t vt = 0, vr = 0;
                     for (uint64_t m = alive; m; m &= m - 1) {
@@ -583,30 +594,30 @@ __device__ __forceinline__ void inst_form(const Ctx &x, Cnt &cn, int i, int base
                     }
                     const int vb = sl_blocks(x, i, p[v]) + (int)((granted >> v) & 1ull);
                     alive &= ~(1ull << v);
-                    x.free_[i] = fr;
+                    x.free_[i] = fb;
                     preempt_book(x, cn, i, p[v], vb);
-                    fr = x.free_[i];
+                    fb = x.free_[i];
                     if (v == q) break;
                 }
             }
-            x.free_[i] = fr;
+            x.free_[i] = fb;
             int w = 0;
             for (int q = 0; q < n; ++q)
                 if ((alive >> q) & 1ull) { if (w != q) p[w] = p[q]; ++w; }
             x.nrun[i] = (uint8_t)w;
             recompute_minfin(x, i);
+            n = w;  // preemptions changed the free blocks, queues and head of line
+            fr = x.free_[i];
+            wm = x.wmask[i];
+            need = x.hol[i];
         }
     }
     // (ii) admission
-    n = x.nrun[i];
     const int n_decode = n;
-    int fr = x.free_[i];
     int prefill = 0;
     int nfresh = 0;  // admitted requests without a token yet: their first token ends this iteration
     while (n < x.Bmax) {
-        const uint32_t wm = x.wmask[i];
         if (!wm) break;
-        const int need = x.hol[i];
         if (need > fr) break;
         const int k = __ffs(wm) - 1;
         const uint32_t info = x.hinfo[i * x.K + k];
@@ -616,7 +627,7 @@ __device__ __forceinline__ void inst_form(const Ctx &x, Cnt &cn, int i, int base
         const uint32_t r = pop_front(x, i, k, cn.status);
         if (r == kNone) break;
         const uint32_t c = info & 0xFFFFu;
-        slot_join(x, i, n, r, c, info >> 16, (uint32_t)k);
+        slot_join_at(x, i, n, r, c, info >> 16, (uint32_t)k, nf, ph);
         if (ft == kNone) {
             slot_ptr(x, i, n)->w |= kFreshFlag;
             ++nfresh;
@@ -625,6 +636,8 @@ __device__ __forceinline__ void inst_form(const Ctx &x, Cnt &cn, int i, int base
         fr -= need;
         prefill += (int)c;
         refresh_hol(x, i);
+        wm = x.wmask[i];
+        need = x.hol[i];
     }
     x.nrun[i] = (uint8_t)n;
     x.free_[i] = fr;
@@ -647,8 +660,8 @@ __device__ __forceinline__ void inst_form(const Ctx &x, Cnt &cn, int i, int base
             }
             cn.events += (uint64_t)nfresh;
         }
-        x.nf[i] += 1u;
-        x.phase[i] = x.phase[i] + 1u == (uint32_t)x.T ? (uint8_t)0 : (uint8_t)(x.phase[i] + 1u);
+        x.nf[i] = nf + 1u;
+        x.phase[i] = ph + 1u == (uint32_t)x.T ? (uint8_t)0 : (uint8_t)(ph + 1u);
         x.pc[i] = 0;
         cn.iterations++;
         cn.member_iterations += (uint64_t)n;
