@@ -470,26 +470,33 @@ __device__ __forceinline__ uint32_t solo_finish(const Ctx &x, Cnt &cn, int i) {
     const int n = x.nrun[i];
     const uint32_t nf = x.nf[i];
     uint4 *p = slot_ptr(x, i, 0);
-    int w = 0, freed = 0;
-    uint32_t fm = kNone, nfin = 0;
+    // a pass of loads only: which records finish, the blocks they free, the
+    // next finishing formation of the others
+    uint64_t fmask = 0;
+    uint32_t fm = kNone;
+    int freed = 0;
     for (int q = 0; q < n; ++q) {
         const uint4 sl = p[q];
         const uint32_t fin = sl_fin(sl);
-        if (fin == nf) {
-            x.res[sl.x].finish_us = x.t;
-            x.res[sl.x].final_instance = (uint16_t)i;
-            freed += blocks_for(x, sl_c(sl) + nf - sl.y);
-            cnt_dec(x, i, (int)sl_tier(sl));
-            x.hist[i * x.TH + sl_rho(sl)]--;
-            ++nfin;
-        } else {
-            if (w != q) p[w] = sl;
-            ++w;
-            fm = min(fm, fin);
-        }
+        const bool f = fin == nf;
+        fmask |= (uint64_t)f << q;
+        fm = f ? fm : min(fm, fin);
+        freed += f ? blocks_for(x, sl_c(sl) + nf - sl.y) : 0;
     }
+    const uint32_t nfin = (uint32_t)__popcll((long long)fmask);
+    for (uint64_t m = fmask; m; m &= m - 1) {
+        const uint4 sl = p[__ffsll((long long)m) - 1];
+        x.res[sl.x].finish_us = x.t;
+        x.res[sl.x].final_instance = (uint16_t)i;
+        cnt_dec(x, i, (int)sl_tier(sl));
+        x.hist[i * x.TH + sl_rho(sl)]--;
+    }
+    // keep the others in order, from the first finished position on
+    int w = fmask ? __ffsll((long long)fmask) - 1 : n;
+    for (int q = w + 1; q < n; ++q)
+        if (!((fmask >> q) & 1ull)) p[w++] = p[q];
     x.free_[i] += freed;
-    x.nrun[i] = (uint8_t)w;
+    x.nrun[i] = (uint8_t)(n - (int)nfin);
     x.minfin[i] = fm;
     cn.events += nfin;
     return nfin;
