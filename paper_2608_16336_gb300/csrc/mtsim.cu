@@ -88,7 +88,6 @@ enum : int { MIG_NONE = 0, MIG_SRC = 1, MIG_DST = 2 };
 // requests that need a new block at the next formation is the count of
 // running requests with rho == -nf (mod T), and a request finishes at the
 // iteration that follows formation phi + left - 1.
-constexpr uint32_t kFreshFlag = 1u << 8;  // set between admission and the end of formation: no token yet
 
 // A waiting request's queue node (16 bytes, indexed by request) carries what
 // admitting it needs: x = next, y = info of next, z = prev, w = own info, with
@@ -622,23 +621,15 @@ __device__ __forceinline__ void inst_form(const Ctx &x, Cnt &cn, int i, int base
     // (ii) admission
     const int n_decode = n;
     int prefill = 0;
-    int nfresh = 0;  // admitted requests without a token yet: their first token ends this iteration
     while (n < x.Bmax) {
         if (!wm) break;
         if (need > fr) break;
         const int k = __ffs(wm) - 1;
         const uint32_t info = x.hinfo[i * x.K + k];
-        const uint32_t h = x.head[i * x.K + k];
-        // issued before the node read so that the two loads overlap
-        const uint32_t ft = x.res[min(h, x.Q - 1u)].first_token_us;
         const uint32_t r = pop_front(x, i, k, cn.status);
         if (r == kNone) break;
         const uint32_t c = info & 0xFFFFu;
         slot_join_at(x, i, n, r, c, info >> 16, (uint32_t)k, nf, ph);
-        if (ft == kNone) {
-            slot_ptr(x, i, n)->w |= kFreshFlag;
-            ++nfresh;
-        }
         ++n;
         fr -= need;
         prefill += (int)c;
@@ -656,17 +647,8 @@ __device__ __forceinline__ void inst_form(const Ctx &x, Cnt &cn, int i, int base
             return;
         }
         x.busy[i] = (uint32_t)end;
-        if (nfresh) {
-            uint4 *sp = slot_ptr(x, i, 0);
-            for (int q = n_decode; q < n; ++q) {
-                const uint4 sl = sp[q];
-                if (sl.w & kFreshFlag) {
-                    x.res[sl.x].first_token_us = (uint32_t)end;
-                    sp[q].w = sl.w & ~kFreshFlag;
-                }
-            }
-            cn.events += (uint64_t)nfresh;
-        }
+        const uint4 *sp = slot_ptr(x, i, 0);
+        for (int q = n_decode; q < n; ++q) atomicMin(&x.res[sp[q].x].first_token_us, (uint32_t)end);
         x.nf[i] = nf + 1u;
         x.phase[i] = ph + 1u == (uint32_t)x.T ? (uint8_t)0 : (uint8_t)(ph + 1u);
         x.pc[i] = 0;
@@ -1323,7 +1305,29 @@ __global__ void k_validate(const long long *offsets, int R, const uint32_t *arri
     }
 }
 
-__global__ void k_export_stats(const RepState *rep, sim_replica_stats_t *out, int R, int *unfinished) {
+// Per replica, the number of requests that have a first token; the simulation
+// kernel records first tokens without counting them (see inst_form), so the
+// exported event count adds these.
+__global__ void k_first_tokens(const long long *offsets, int R, const sim_request_result_t *res, uint32_t *count) {
+    __shared__ uint32_t part[32];
+    for (int r = blockIdx.x; r < R; r += gridDim.x) {
+        uint32_t c = 0;
+        for (long long i = offsets[r] + threadIdx.x; i < offsets[r + 1]; i += blockDim.x)
+            c += res[i].first_token_us != kNone ? 1u : 0u;
+        c = __reduce_add_sync(kFull, c);
+        if ((threadIdx.x & 31) == 0) part[threadIdx.x >> 5] = c;
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            uint32_t t = 0;
+            for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += part[w];
+            count[r] = t;
+        }
+        __syncthreads();
+    }
+}
+
+__global__ void k_export_stats(const RepState *rep, sim_replica_stats_t *out, int R, int *unfinished,
+                               const uint32_t *first_tokens) {
     for (int r = blockIdx.x * blockDim.x + threadIdx.x; r < R; r += gridDim.x * blockDim.x) {
         const RepState s = rep[r];
         if (out) {
@@ -1331,7 +1335,7 @@ __global__ void k_export_stats(const RepState *rep, sim_replica_stats_t *out, in
             o.steps = s.steps;
             o.iterations = s.iterations;
             o.member_iterations = s.member_iterations;
-            o.events = s.events;
+            o.events = s.events + (first_tokens ? first_tokens[r] : 0u);
             o.migrations = s.migrations;
             o.preemptions = s.preemptions;
             o.migration_starts = s.starts;
@@ -1477,6 +1481,7 @@ struct sim {
     uint4 *d_node = nullptr;
     sim_request_result_t *d_res = nullptr;
     uint32_t *d_drain = nullptr;  // [R][N] drain start times (sim_set_drain), or NULL
+    uint32_t *d_ftc = nullptr;    // [R] first-token counts for sim_metrics
     sim_latency_stats_t *d_lat = nullptr;  // device staging of sim_latency_stats for host output
     int *d_lat_rep = nullptr;              // chunk table of sim_latency_stats: replica and first record
     long long *d_lat_b0 = nullptr;
@@ -1920,7 +1925,7 @@ int sim_run(sim_t *s, int64_t max_steps, int64_t *num_unfinished) {
         e = cudaMemsetAsync(s->d_work + 2, 0, 4, s->stream);
         if (e != cudaSuccess) return cuda_fail(s, e, "sim_run");
         const int R = s->cl.num_replicas;
-        mt::k_export_stats<<<(R + 255) / 256, 256, 0, s->stream>>>(s->d_rep, nullptr, R, s->d_work + 2);
+        mt::k_export_stats<<<(R + 255) / 256, 256, 0, s->stream>>>(s->d_rep, nullptr, R, s->d_work + 2, nullptr);
         rc = check_launch(s, "k_export_stats");
         if (rc) return rc;
         e = cudaMemcpyAsync(&cnt, s->d_work + 2, 4, cudaMemcpyDeviceToHost, s->stream);
@@ -1948,8 +1953,15 @@ int sim_metrics(sim_t *s, sim_request_result_t *per_request, sim_replica_stats_t
             if (!tmp) return fail(s, SIM_ERR_OOM, "device allocation failed");
             dst = tmp;
         }
-        mt::k_export_stats<<<(R + 255) / 256, 256, 0, s->stream>>>(s->d_rep, dst, R, nullptr);
-        int rc = check_launch(s, "k_export_stats");
+        if (!s->d_ftc) {
+            s->d_ftc = (uint32_t *)dalloc(s, (size_t)R * 4);
+            if (!s->d_ftc) return fail(s, SIM_ERR_OOM, "device allocation failed");
+        }
+        mt::k_first_tokens<<<std::max(1, std::min(R, s->sms * 8)), 256, 0, s->stream>>>(s->d_off, R, s->d_res, s->d_ftc);
+        int rc = check_launch(s, "k_first_tokens");
+        if (rc) return rc;
+        mt::k_export_stats<<<(R + 255) / 256, 256, 0, s->stream>>>(s->d_rep, dst, R, nullptr, s->d_ftc);
+        rc = check_launch(s, "k_export_stats");
         if (rc) return rc;
         if (tmp) {
             e = cudaMemcpyAsync(per_replica, tmp, (size_t)R * sizeof(sim_replica_stats_t), cudaMemcpyDeviceToHost,
@@ -2025,6 +2037,7 @@ extern "C" int sim_run_static(const sim_cluster_t *cl, const sim_tier_table_t *t
     const size_t o_tk = o; o = align256(o + (size_t)tt->num_tables * 4);
     const size_t o_th = o; o = align256(o + (size_t)tt->num_tables * K * 4);
     const size_t o_work = o; o = align256(o + 16);
+    const size_t o_ftc = o; o = align256(o + (size_t)R * 4);
     if (o > (size_t)SIM_STATIC_SCRATCH_BYTES)
         return fail(nullptr, SIM_ERR_ARG, "problem needs %zu bytes of scratch; sim_run_static holds %u bytes", o,
                     (unsigned)SIM_STATIC_SCRATCH_BYTES);
@@ -2101,7 +2114,9 @@ extern "C" int sim_run_static(const sim_cluster_t *cl, const sim_tier_table_t *t
         lc.fn_ext<<<lc.grid_ext, 32 * mt::kWarpsPerBlock, lc.smem, st>>>(p);
     else
         lc.fn<<<lc.grid, 32 * mt::kWarpsPerBlock, lc.smem, st>>>(p);
-    mt::k_export_stats<<<(R + 255) / 256, 256, 0, st>>>(p.rep, per_replica, R, nullptr);
+    uint32_t *ftc = (uint32_t *)(base + o_ftc);
+    mt::k_first_tokens<<<std::max(1, std::min(R, sms * 8)), 256, 0, st>>>(p.offsets, R, per_request, ftc);
+    mt::k_export_stats<<<(R + 255) / 256, 256, 0, st>>>(p.rep, per_replica, R, nullptr, ftc);
     e = cudaGetLastError();
     if (e == cudaSuccess) e = cudaStreamSynchronize(st);
     if (e != cudaSuccess) return fail(nullptr, SIM_ERR_CUDA, "sim_run_static: %s", cudaGetErrorString(e));
