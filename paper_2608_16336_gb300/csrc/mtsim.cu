@@ -664,13 +664,28 @@ __device__ __forceinline__ void dispatch_one(const Ctx &x, Cnt &cn, uint32_t r, 
                                              uint32_t all) {
     const int best = arg_ext<C>(x, all, true, -1);
     if (x.lane == 0) {
+        // the destination's scalars, read together; the new key is computed from them
+        const int b = best * x.K + k;
         const uint32_t old = x.wmask[best];
-        push_back(x, best, k, r, P | (O << 16));
-        cnt_inc(x, best, k);
-        if ((old & ((2u << k) - 1u)) == 0) x.hol[best] = blocks_for(x, P);  // becomes head of line
+        const uint32_t tl = x.tail[b];
+        const uint32_t c0 = x.cnt[b];
+        int hol = x.hol[best];
+        int hr = x.hr[best];
+        const int fr = x.free_[best];
+        const int nr = x.nrun[best];
+        const int hk = x.h[k];
+        const uint32_t info = P | (O << 16);
+        x.node[r] = make_uint4(kNone, 0u, tl, info);  // appended to bucket (best, k), as push_back
+        if (tl != kNone) *reinterpret_cast<uint2 *>(&x.node[tl]) = make_uint2(r, info);
+        else { x.head[b] = r; x.hinfo[b] = info; }
+        x.tail[b] = r;
+        x.wmask[best] = (uint16_t)(old | (1u << k));
+        x.cnt[b] = (uint16_t)(c0 + 1u);
+        if (c0 == 0) x.hr[best] = hr += hk;                    // tier k now present (Eq. 4)
+        if ((old & ((2u << k) - 1u)) == 0) x.hol[best] = hol = blocks_for(x, P);  // becomes head of line
         x.res[r].dispatch_instance = (uint16_t)best;
         cn.events++;
-        set_key(x, best);
+        x.key[best] = make_key(x, fr - hol - hr, nr);
     }
     __syncwarp();
 }
