@@ -473,20 +473,21 @@ __device__ __forceinline__ uint32_t solo_finish(const Ctx &x, Cnt &cn, int i) {
     // next finishing formation of the others
     uint64_t fmask = 0;
     uint32_t fm = kNone;
-    int freed = 0;
+#pragma unroll 4
     for (int q = 0; q < n; ++q) {
         const uint4 sl = p[q];
         const uint32_t fin = sl_fin(sl);
         const bool f = fin == nf;
         fmask |= (uint64_t)f << q;
         fm = f ? fm : min(fm, fin);
-        freed += f ? blocks_for(x, sl_c(sl) + nf - sl.y) : 0;
     }
     const uint32_t nfin = (uint32_t)__popcll((long long)fmask);
+    int freed = 0;
     for (uint64_t m = fmask; m; m &= m - 1) {
         const uint4 sl = p[__ffsll((long long)m) - 1];
         x.res[sl.x].finish_us = x.t;
         x.res[sl.x].final_instance = (uint16_t)i;
+        freed += blocks_for(x, sl_c(sl) + nf - sl.y);
         cnt_dec(x, i, (int)sl_tier(sl));
         x.hist[i * x.TH + sl_rho(sl)]--;
     }
