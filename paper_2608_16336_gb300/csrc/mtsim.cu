@@ -583,11 +583,12 @@ __device__ __forceinline__ void inst_form(const Ctx &x, Cnt &cn, int i, int base
             uint4 *p = slot_ptr(x, i, 0);
             const uint64_t all = n >= 64 ? ~0ull : ((1ull << n) - 1ull);
             uint64_t alive = all, needs = 0, granted = 0;
-            for (int q = 0; q < n; ++q) {
-                const uint4 sl = p[q];
-                if (blocks_for(x, sl_c(sl) + sl_adv(x, i, sl)) > sl_blocks(x, i, sl)) needs |= 1ull << q;
-            }
-            int fb = x.free_[i];
+            // The requests that need a block now are those whose context reaches
+            // a block boundary: rho == -nf (mod T), the ones hist counts.
+            const uint32_t target = ph == 0 ? 0u : (uint32_t)x.T - ph;
+#pragma unroll 4
+            for (int q = 0; q < n; ++q) needs |= (uint64_t)(sl_rho(p[q]) == target) << q;
+            int fb = fr;
             for (int q = 0; q < n; ++q) {
                 if (!((alive & needs) >> q & 1ull)) continue;
                 for (;;) {
@@ -599,7 +600,7 @@ __device__ __forceinline__ void inst_form(const Ctx &x, Cnt &cn, int i, int base
                         const uint32_t ts = sl_tier(p[s2]), rs = p[s2].x;
                         if (v < 0 || ts > vt || (ts == vt && rs > vr)) { v = s2; vt = ts; vr = rs; }
                     }
-                    const int vb = sl_blocks(x, i, p[v]) + (int)((granted >> v) & 1ull);
+                    const int vb = blocks_for(x, sl_c(p[v]) + nf - p[v].y) + (int)((granted >> v) & 1ull);
                     alive &= ~(1ull << v);
                     x.free_[i] = fb;
                     preempt_book(x, cn, i, p[v], vb);
@@ -609,10 +610,17 @@ __device__ __forceinline__ void inst_form(const Ctx &x, Cnt &cn, int i, int base
             }
             x.free_[i] = fb;
             int w = 0;
-            for (int q = 0; q < n; ++q)
-                if ((alive >> q) & 1ull) { if (w != q) p[w] = p[q]; ++w; }
+            uint32_t fm = kNone;  // the survivors' next finishing formation
+            for (int q = 0; q < n; ++q) {
+                if ((alive >> q) & 1ull) {
+                    const uint4 sl = p[q];
+                    if (w != q) p[w] = sl;
+                    ++w;
+                    fm = min(fm, sl_fin(sl));
+                }
+            }
             x.nrun[i] = (uint8_t)w;
-            recompute_minfin(x, i);
+            x.minfin[i] = fm;
             n = w;  // preemptions changed the free blocks, queues and head of line
             fr = x.free_[i];
             wm = x.wmask[i];
