@@ -460,48 +460,6 @@ __device__ __forceinline__ void coop_finish(const Ctx &x, Cnt &cn, int i) {
     __syncwarp();
 }
 
-// Phase 1, second part, one lane: the requests of instance i whose output is
-// complete finish at x.t and free their KV, for an instance in no migration
-// (so nothing outside instance i changes).  The owner lane scans its slots
-// (independent loads) and compacts them in order.  Returns how many finished;
-// the caller adds them to the replica's count.
-__device__ __forceinline__ uint32_t solo_finish(const Ctx &x, Cnt &cn, int i) {
-    const int n = x.nrun[i];
-    const uint32_t nf = x.nf[i];
-    uint4 *p = slot_ptr(x, i, 0);
-    // a pass of loads only: which records finish, the blocks they free, the
-    // next finishing formation of the others
-    uint64_t fmask = 0;
-    uint32_t fm = kNone;
-#pragma unroll 4
-    for (int q = 0; q < n; ++q) {
-        const uint4 sl = p[q];
-        const uint32_t fin = sl_fin(sl);
-        const bool f = fin == nf;
-        fmask |= (uint64_t)f << q;
-        fm = f ? fm : min(fm, fin);
-    }
-    const uint32_t nfin = (uint32_t)__popcll((long long)fmask);
-    int freed = 0;
-    for (uint64_t m = fmask; m; m &= m - 1) {
-        const uint4 sl = p[__ffsll((long long)m) - 1];
-        x.res[sl.x].finish_us = x.t;
-        x.res[sl.x].final_instance = (uint16_t)i;
-        freed += blocks_for(x, sl_c(sl) + nf - sl.y);
-        cnt_dec(x, i, (int)sl_tier(sl));
-        x.hist[i * x.TH + sl_rho(sl)]--;
-    }
-    // keep the others in order, from the first finished position on
-    int w = fmask ? __ffsll((long long)fmask) - 1 : n;
-    for (int q = w + 1; q < n; ++q)
-        if (!((fmask >> q) & 1ull)) p[w++] = p[q];
-    x.free_[i] += freed;
-    x.nrun[i] = (uint8_t)(n - (int)nfin);
-    x.minfin[i] = fm;
-    cn.events += nfin;
-    return nfin;
-}
-
 // One copy stage at the end of an iteration of migration source s, whole
 // warp: up to S of the request's blocks are reserved on the destination
 // (abandoning the migration if they do not fit), and the request commits
@@ -1136,7 +1094,7 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
                 }
                 uint32_t fresh = 0;  // distinct event times this lane contributes (C > 1)
                 uint32_t tlast = 0;  // latest event time processed in the window
-                uint32_t sfin = 0;   // requests this lane's instances finished in the window
+                uint32_t fz = 0;     // this lane's instances with a finishing request
 #pragma unroll
                 for (int j = 0; j < C; ++j) {
                     if (!((solo >> j) & 1u)) continue;
@@ -1144,8 +1102,24 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
                     x.t = bz[j];
                     tlast = max(tlast, bz[j]);
                     if (C > 1) fresh += tset_insert(x, bz[j]);
-                    if (inst_complete_head(x, i)) sfin += solo_finish(x, cn, i);
-                    inst_form(x, cn, i, p.base, p.a, p.b);
+                    if (inst_complete_head(x, i)) fz |= 1u << j;
+                }
+                // finishes, one instance at a time by the whole warp (they touch
+                // only their own instance, so their order does not matter) ...
+                for (uint32_t fl = __ballot_sync(kFull, fz != 0); fl; fl &= fl - 1) {
+                    const int l = __ffs(fl) - 1;
+                    for (uint32_t h = C == 1 ? 1u : __shfl_sync(kFull, fz, l); h; h &= h - 1) {
+                        const int j = __ffs(h) - 1;
+                        x.t = __shfl_sync(kFull, bz[j], l);
+                        coop_finish(x, cn, l * C + j);
+                    }
+                }
+                // ... then every lane forms its instances' next batches together
+#pragma unroll
+                for (int j = 0; j < C; ++j) {
+                    if (!((solo >> j) & 1u)) continue;
+                    x.t = bz[j];
+                    inst_form(x, cn, lane * C + j, p.base, p.a, p.b);
                 }
                 __syncwarp();
                 uint32_t ucount, u = kNone;
@@ -1188,8 +1162,7 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
                 }
                 cn.steps += ucount;
                 x.t = __reduce_max_sync(kFull, tlast);
-                // lane 0 counted the finishes of steps in time order; the lanes, their own
-                cn.finished = __shfl_sync(kFull, cn.finished, 0) + __reduce_add_sync(kFull, sfin);
+                cn.finished = __shfl_sync(kFull, cn.finished, 0);  // finishes are all counted on lane 0
                 const int ws = __reduce_min_sync(kFull, cn.status);
                 cn.status = ws;
                 if (cn.status < 0) break;
