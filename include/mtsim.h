@@ -137,14 +137,15 @@ typedef struct {
 
 /* Per-request outcome, 16 bytes.  Times are microseconds from the replica's
  * start; TTFT = first_token_us - arrival, E2E = finish_us - arrival.  The
- * migration and preemption counters are kept modulo 2^16. */
+ * preemption and migration counters are kept modulo 2^16 (each exactly: they
+ * share the last 32-bit word, preemptions in the low half). */
 typedef struct {
     uint16_t dispatch_instance;  /* instance chosen at arrival (SIM_NONE16 if not yet arrived) */
     uint16_t final_instance;     /* instance it finished on (SIM_NONE16 if unfinished) */
     uint32_t first_token_us;     /* SIM_NONE32 if no token yet */
     uint32_t finish_us;          /* SIM_NONE32 if unfinished */
-    uint16_t n_migrations;       /* queued moves + committed running migrations */
     uint16_t n_preemptions;
+    uint16_t n_migrations;       /* queued moves + committed running migrations */
 } sim_request_result_t;
 
 typedef struct {

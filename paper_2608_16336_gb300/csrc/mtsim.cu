@@ -304,11 +304,18 @@ __device__ __forceinline__ void log_ev(const Ctx &x, Cnt &cn, int kind, uint32_t
         reinterpret_cast<uint4 *>(x.log)[k] = w;
     }
 }
-__device__ __forceinline__ void bump_mig(const Ctx &x, uint32_t r) {
-    atomicAdd(reinterpret_cast<unsigned int *>(reinterpret_cast<unsigned char *>(x.res + r) + 12), 1u);
+// The result record's last word holds n_preemptions (low half) and
+// n_migrations (high half), both modulo 2^16.  A migration adds 1 << 16: a
+// wrap carries out of the word, so nothing waits on the add.  A preemption
+// adds 1 to the low half and gets the old word back; when the low half
+// wrapped, the carry into n_migrations is taken back (pre_fix).
+__device__ __forceinline__ unsigned int *count_word(const Ctx &x, uint32_t r) {
+    return reinterpret_cast<unsigned int *>(reinterpret_cast<unsigned char *>(x.res + r) + 12);
 }
-__device__ __forceinline__ void bump_pre(const Ctx &x, uint32_t r) {
-    atomicAdd(reinterpret_cast<unsigned int *>(reinterpret_cast<unsigned char *>(x.res + r) + 12), 1u << 16);
+__device__ __forceinline__ void bump_mig(const Ctx &x, uint32_t r) { atomicAdd(count_word(x, r), 1u << 16); }
+__device__ __forceinline__ unsigned int bump_pre(const Ctx &x, uint32_t r) { return atomicAdd(count_word(x, r), 1u); }
+__device__ __forceinline__ void pre_fix(const Ctx &x, uint32_t r, unsigned int old) {
+    if ((old & 0xFFFFu) == 0xFFFFu) atomicSub(count_word(x, r), 1u << 16);
 }
 __device__ __forceinline__ void clear_mig(const Ctx &x, int s, int d) {
     x.mrole[s] = MIG_NONE;
@@ -500,7 +507,7 @@ __device__ __forceinline__ void coop_stage(const Ctx &x, Cnt &cn, int s) {
 // Recompute-style preemption of running request `sl` (holding `blocks` KV
 // blocks) on instance i: its KV is freed, it keeps its generated tokens and
 // goes back to the front of its tier's bucket.  The caller drops its slot.
-__device__ __forceinline__ void preempt_book(const Ctx &x, Cnt &cn, int i, const uint4 &sl, int blocks) {
+__device__ __forceinline__ unsigned int preempt_book(const Ctx &x, Cnt &cn, int i, const uint4 &sl, int blocks) {
     const uint32_t r = sl.x;
     const int tr = (int)sl_tier(sl);
     const uint32_t adv = sl_adv(x, i, sl);
@@ -509,10 +516,11 @@ __device__ __forceinline__ void preempt_book(const Ctx &x, Cnt &cn, int i, const
     push_front(x, i, tr, r, (sl_c(sl) + adv) | ((sl_left(sl) - adv) << 16));
     if ((old & ((1u << tr) - 1u)) == 0) x.hol[i] = blocks_for(x, sl_c(sl) + adv);  // now head of line
     x.hist[i * x.TH + sl_rho(sl)]--;
-    bump_pre(x, r);
+    const unsigned int word = bump_pre(x, r);
     cn.preemptions++;
     cn.events++;
     if (x.mrole[i] == MIG_SRC && x.mreq[i] == r) abort_mig(x, cn, i);
+    return word;  // for pre_fix, which the caller runs later so that nothing waits here
 }
 
 // Phase 4: batch formation at idle instance i at x.t (Sec. 2.2, Sec. 3.1):
@@ -544,24 +552,41 @@ __device__ __forceinline__ void inst_form(const Ctx &x, Cnt &cn, int i, int base
             // The requests that need a block now are those whose context reaches
             // a block boundary: rho == -nf (mod T), the ones hist counts.
             const uint32_t target = ph == 0 ? 0u : (uint32_t)x.T - ph;
+            // the same pass finds the first victim (lowest priority, then newest):
+            // more requests need a block than there are free blocks, so there is one
+            int v1 = -1;
+            uint32_t vt1 = 0, vr1 = 0;
 #pragma unroll 4
-            for (int q = 0; q < n; ++q) needs |= (uint64_t)(sl_rho(p[q]) == target) << q;
+            for (int q = 0; q < n; ++q) {
+                const uint4 sl = p[q];
+                needs |= (uint64_t)(sl_rho(sl) == target) << q;
+                const uint32_t ts = sl_tier(sl);
+                if (v1 < 0 || ts > vt1 || (ts == vt1 && sl.x > vr1)) { v1 = q; vt1 = ts; vr1 = sl.x; }
+            }
             int fb = fr;
+            uint32_t pr = kNone;  // the last preempted request and its counter word before the add
+            unsigned int pold = 0;
             for (int q = 0; q < n; ++q) {
                 if (!((alive & needs) >> q & 1ull)) continue;
                 for (;;) {
                     if (fb > 0) { --fb; granted |= 1ull << q; break; }
                     int v = -1;
-                    uint32_t vt = 0, vr = 0;
-                    for (uint64_t m = alive; m; m &= m - 1) {
-                        const int s2 = __ffsll((long long)m) - 1;
-                        const uint32_t ts = sl_tier(p[s2]), rs = p[s2].x;
-                        if (v < 0 || ts > vt || (ts == vt && rs > vr)) { v = s2; vt = ts; vr = rs; }
+                    if (alive == all) {
+                        v = v1;  // nobody preempted yet: the victim found by the scan
+                    } else {
+                        uint32_t vt = 0, vr = 0;
+                        for (uint64_t m = alive; m; m &= m - 1) {
+                            const int s2 = __ffsll((long long)m) - 1;
+                            const uint32_t ts = sl_tier(p[s2]), rs = p[s2].x;
+                            if (v < 0 || ts > vt || (ts == vt && rs > vr)) { v = s2; vt = ts; vr = rs; }
+                        }
                     }
                     const int vb = blocks_for(x, sl_c(p[v]) + nf - p[v].y) + (int)((granted >> v) & 1ull);
                     alive &= ~(1ull << v);
                     x.free_[i] = fb;
-                    preempt_book(x, cn, i, p[v], vb);
+                    if (pr != kNone) pre_fix(x, pr, pold);
+                    pr = p[v].x;
+                    pold = preempt_book(x, cn, i, p[v], vb);
                     fb = x.free_[i];
                     if (v == q) break;
                 }
@@ -579,6 +604,7 @@ __device__ __forceinline__ void inst_form(const Ctx &x, Cnt &cn, int i, int base
             }
             x.nrun[i] = (uint8_t)w;
             x.minfin[i] = fm;
+            if (pr != kNone) pre_fix(x, pr, pold);
             n = w;  // preemptions changed the free blocks, queues and head of line
             fr = x.free_[i];
             wm = x.wmask[i];

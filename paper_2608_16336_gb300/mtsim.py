@@ -26,7 +26,7 @@ SIM_NONE32, SIM_NONE16 = 0xFFFFFFFF, 0xFFFF
 SIM_MAX_TIERS = 16
 
 RESULT_DTYPE = np.dtype([("dispatch_instance", "<u2"), ("final_instance", "<u2"), ("first_token_us", "<u4"),
-                         ("finish_us", "<u4"), ("n_migrations", "<u2"), ("n_preemptions", "<u2")])
+                         ("finish_us", "<u4"), ("n_preemptions", "<u2"), ("n_migrations", "<u2")])
 STATS_DTYPE = np.dtype([("steps", "<u8"), ("iterations", "<u8"), ("member_iterations", "<u8"), ("events", "<u8"),
                         ("migrations", "<u4"), ("preemptions", "<u4"), ("migration_starts", "<u4"),
                         ("migration_aborts", "<u4"), ("log_events", "<u4"), ("finished", "<u4"),
