@@ -722,7 +722,14 @@ __device__ __forceinline__ void dispatch_phase(const Ctx &x, Cnt &cn, uint32_t &
         arr_refill(x, ab, cursor);
         eq = __ballot_sync(kFull, ab.time == x.t);
     }
-    if (eq != kFull) {
+    if (eq != kFull && (eq & (eq - 1u)) == 0u) {
+        // one arrival at t (the usual case): no tier ordering to do
+        const int l = __ffs(eq) - 1;
+        const uint32_t k1 = __shfl_sync(kFull, ab.tier, l);
+        const uint32_t po = __shfl_sync(kFull, ab.P | (ab.O << 16), l);
+        dispatch_one<C>(x, cn, ab.pb + (uint32_t)l, (int)k1, po & 0xFFFFu, po >> 16, all);
+        cursor += 1u;
+    } else if (eq != kFull) {
         const bool mine = (eq >> x.lane) & 1u;
         uint32_t tm = __reduce_or_sync(kFull, mine ? (1u << ab.tier) : 0u);
         while (tm) {
@@ -1066,6 +1073,7 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
         x.lane = lane;
         x.drains = EXT ? p.drains : 0;
         x.t = rs.t;
+        uint32_t tmax = rs.t;  // latest event time this lane has processed (the replica's: max over lanes)
         Cnt cn;  // lane 0: the replica's totals; other lanes: what they add in windows
         const bool l0 = lane == 0;
         cn.finished = rs.finished;
@@ -1187,7 +1195,7 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
                     }
                 }
                 cn.steps += ucount;
-                x.t = __reduce_max_sync(kFull, tlast);
+                tmax = max(tmax, tlast);  // x.t is set again before any further use
                 cn.finished = __shfl_sync(kFull, cn.finished, 0);  // finishes are all counted on lane 0
                 const int ws = __reduce_min_sync(kFull, cn.status);
                 cn.status = ws;
@@ -1199,6 +1207,7 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
             if (tc == kNone) { cn.status = SIM_ERR_DEADLOCK; break; }
             const bool tick = ticks && next_tick <= tc;
             x.t = tick ? next_tick : tc;
+            tmax = max(tmax, x.t);
             ++cn.steps;
             const uint32_t f1 = cn.finished;
             if (tb == x.t) complete_all<C>(x, cn, all);  // 1. iteration ends
@@ -1217,6 +1226,7 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
         }
         __syncwarp();
         // fold the other lanes' counters into lane 0's
+        const uint32_t tfin = __reduce_max_sync(kFull, tmax);
         const uint32_t a_pre = __reduce_add_sync(kFull, l0 ? 0u : cn.preemptions);
         const uint32_t a_it = __reduce_add_sync(kFull, cn.iterations);
         uint64_t a_mi = cn.member_iterations, a_ev = cn.events;
@@ -1231,7 +1241,7 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
                    slot_bytes, lane);
         if (l0) {
             RepState o2;
-            o2.t = x.t;
+            o2.t = tfin;
             o2.cursor = cursor;
             o2.finished = cn.finished;
             o2.log_events = cn.log_events;
