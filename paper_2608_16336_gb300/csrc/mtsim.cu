@@ -1019,7 +1019,11 @@ __device__ __forceinline__ void form_all(const Ctx &x, Cnt &cn, uint32_t mask, c
 // oracle's order.  EXT: the variant that also handles draining instances and
 // the auto-scaling signal (the other variant compiles that code out).
 template <int C, bool SMS, bool EXT>
-__global__ void __launch_bounds__(32 * kWarpsPerBlock, 4) k_run(Params p) {
+// Variants that keep the running-request records in HBM run workloads with
+// many replicas; asking for 8 resident blocks per SM (at most 128 registers)
+// hides more of their latency.  The others keep 4: their shared memory or
+// register needs limit residency anyway.
+__global__ void __launch_bounds__(32 * kWarpsPerBlock, (!SMS && C <= 2) ? 8 : 4) k_run(Params p) {
     extern __shared__ __align__(16) unsigned char smem[];
     unsigned long long *magic = reinterpret_cast<unsigned long long *>(smem);
     for (int d = threadIdx.x; d <= 64; d += blockDim.x)
