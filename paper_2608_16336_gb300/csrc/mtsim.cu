@@ -651,11 +651,11 @@ __device__ __forceinline__ void inst_form(const Ctx &x, Cnt &cn, int i, int base
 }
 
 // ---- cooperative steps ----------------------------------------------------------
-// Dispatch one arriving request r of tier k with prompt length P (Sec. 3.4).
-template <int C>
-__device__ __forceinline__ void dispatch_one(const Ctx &x, Cnt &cn, uint32_t r, int k, uint32_t P, uint32_t O,
-                                             uint32_t all) {
-    const int best = arg_ext<C>(x, all, true, -1);
+// Lane 0 appends arriving request r (tier k, prompt P, output O) to instance
+// best's bucket and updates the instance (Sec. 3.4); the key store is needed
+// only if another arrival at the same time is dispatched next.
+__device__ __forceinline__ void dispatch_to(const Ctx &x, Cnt &cn, int best, uint32_t r, int k, uint32_t P,
+                                            uint32_t O, bool store_key) {
     if (x.lane == 0) {
         // the destination's scalars, read together; the new key is computed from them
         const int b = best * x.K + k;
@@ -678,8 +678,16 @@ __device__ __forceinline__ void dispatch_one(const Ctx &x, Cnt &cn, uint32_t r, 
         if ((old & ((2u << k) - 1u)) == 0) x.hol[best] = hol = blocks_for(x, P);  // becomes head of line
         x.res[r].dispatch_instance = (uint16_t)best;
         cn.events++;
-        x.key[best] = make_key(x, fr - hol - hr, nr);
+        if (store_key) x.key[best] = make_key(x, fr - hol - hr, nr);
     }
+}
+
+// Dispatch one arriving request r of tier k with prompt length P (Sec. 3.4).
+template <int C>
+__device__ __forceinline__ void dispatch_one(const Ctx &x, Cnt &cn, uint32_t r, int k, uint32_t P, uint32_t O,
+                                             uint32_t all) {
+    const int best = arg_ext<C>(x, all, true, -1);
+    dispatch_to(x, cn, best, r, k, P, O, true);
     __syncwarp();
 }
 
@@ -703,7 +711,6 @@ __device__ __forceinline__ void arr_refill(const Ctx &x, ArrBuf &ab, uint32_t cu
 template <int C, bool EXT>
 __device__ __forceinline__ void dispatch_phase(const Ctx &x, Cnt &cn, uint32_t &cursor, uint32_t &next_arr,
                                                ArrBuf &ab) {
-    refresh_keys<C>(x);
     uint32_t all = own_mask<C>(x);
     if (EXT && x.drains) {
         // Draining instances (infinite virtual usage, Sec. 3.5) get no
@@ -727,9 +734,25 @@ __device__ __forceinline__ void dispatch_phase(const Ctx &x, Cnt &cn, uint32_t &
         const int l = __ffs(eq) - 1;
         const uint32_t k1 = __shfl_sync(kFull, ab.tier, l);
         const uint32_t po = __shfl_sync(kFull, ab.P | (ab.O << 16), l);
-        dispatch_one<C>(x, cn, ab.pb + (uint32_t)l, (int)k1, po & 0xFFFFu, po >> 16, all);
+        // the freest instance from keys computed in registers (nothing reads
+        // the key array before the next refresh)
+        int bv = INT_MIN, bi = -1;
+#pragma unroll
+        for (int j = 0; j < C; ++j) {
+            const int i = x.lane * C + j;
+            if ((all >> j) & 1u) {
+                const int kk = make_key(x, fnum(x, i), x.nrun[i]);
+                if (bi < 0 || kk > bv) { bv = kk; bi = i; }
+            }
+        }
+        const int m = __reduce_max_sync(kFull, bv);
+        const uint32_t em = __ballot_sync(kFull, bi >= 0 && bv == m);
+        const int best = __shfl_sync(kFull, bi, __ffs(em) - 1);
+        dispatch_to(x, cn, best, ab.pb + (uint32_t)l, (int)k1, po & 0xFFFFu, po >> 16, false);
+        __syncwarp();
         cursor += 1u;
     } else if (eq != kFull) {
+        refresh_keys<C>(x);
         const bool mine = (eq >> x.lane) & 1u;
         uint32_t tm = __reduce_or_sync(kFull, mine ? (1u << ab.tier) : 0u);
         while (tm) {
@@ -747,6 +770,7 @@ __device__ __forceinline__ void dispatch_phase(const Ctx &x, Cnt &cn, uint32_t &
     } else {
         // 32 or more arrivals share this time (the buffer starts at the cursor):
         // count them, then go tier by tier from the trace.
+        refresh_keys<C>(x);
         uint32_t m = 32;
         for (;;) {
             const uint32_t j2 = cursor + m + (uint32_t)x.lane;
