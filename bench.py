@@ -27,6 +27,7 @@ import os
 import statistics
 import subprocess
 import sys
+import tempfile
 import time
 
 HERE = os.path.dirname(os.path.abspath(__file__))
@@ -110,10 +111,10 @@ class ClockSampler:
              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
-    def __init__(self, gpu_index: int):
+    def __init__(self, gpu_index: int, out_dir: str):
         self.gpu = gpu_index
         self.proc = None
-        self.path = os.path.join(HERE, "gpurun_out", "clocks_bench_%d.csv" % gpu_index)
+        self.path = os.path.join(out_dir, "clocks_bench_%d.csv" % gpu_index)
 
     def start(self):
         try:
@@ -183,7 +184,7 @@ def bench_gpu(args):
     torch.cuda.synchronize()
     # per-launch duration of the simulation kernel, on its own stream
     k_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
-    clocks = ClockSampler(local)
+    clocks = ClockSampler(local, args.clocks_dir)
     clocks.start()
     barrier()
     torch.cuda.synchronize()
@@ -387,6 +388,8 @@ def main():
     ap.add_argument("--cpu-replicas", type=int, default=256)
     ap.add_argument("--cpu-replicas-per-step", type=int, default=64)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--clocks-dir", default=os.path.join(tempfile.gettempdir(), "mtsim_bench"),
+                    help="where the raw nvidia-smi clock samples of the timed region are written")
     ap.add_argument("--replicas", type=int, default=0, help="profiling only: first N replicas of the workload")
     ap.add_argument("--requests", type=int, default=None, help="profiling only: requests per replica")
     args = ap.parse_args()

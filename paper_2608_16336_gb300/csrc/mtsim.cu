@@ -265,17 +265,6 @@ __device__ __forceinline__ void push_front(const Ctx &x, int i, int k, uint32_t 
     x.hinfo[b] = info;
     x.wmask[i] |= (uint16_t)(1u << k);
 }
-// Removes the head of bucket (i, k); its info is hinfo before the call.
-__device__ __forceinline__ uint32_t pop_front(const Ctx &x, int i, int k, int &status) {
-    const int b = i * x.K + k;
-    const uint32_t r = x.head[b];
-    if (r >= x.Q) { status = SIM_ERR_INTERNAL; return kNone; }
-    const uint4 nd = x.node[r];
-    x.head[b] = nd.x;
-    if (nd.x != kNone) { x.node[nd.x].z = kNone; x.hinfo[b] = nd.y; }
-    else { x.tail[b] = kNone; x.wmask[i] &= (uint16_t)~(1u << k); }
-    return r;
-}
 // Removes the tail of bucket (i, k) and returns its info in `info`.
 __device__ __forceinline__ uint32_t pop_back(const Ctx &x, int i, int k, uint32_t &info, int &status) {
     const int b = i * x.K + k;
@@ -366,32 +355,17 @@ __device__ __forceinline__ void slot_join(const Ctx &x, int i, int n, uint32_t r
     slot_join_at(x, i, n, r, c, left, tier, x.nf[i], x.phase[i]);
 }
 
-// Removes slot s of instance i's running list (order kept); returns its record.
-__device__ __forceinline__ uint4 slot_remove(const Ctx &x, int i, int s) {
-    uint4 *p = slot_ptr(x, i, 0);
-    const uint4 out = p[s];
-    const int n = x.nrun[i];
-    for (int q = s + 1; q < n; ++q) p[q - 1] = p[q];
-    x.nrun[i] = (uint8_t)(n - 1);
-    x.hist[i * x.TH + sl_rho(out)]--;
-    return out;
-}
-
-__device__ __forceinline__ void recompute_minfin(const Ctx &x, int i) {
-    const uint4 *p = slot_ptr(x, i, 0);
-    uint32_t m = kNone;
-    for (int s = 0, n = x.nrun[i]; s < n; ++s) m = min(m, sl_fin(p[s]));
-    x.minfin[i] = m;
-}
-
-// Commit a fully copied running request (slot pos of source s) to d (Sec. 3.5, Fig. 4).
-__device__ __forceinline__ void commit_mig(const Ctx &x, Cnt &cn, int s, int pos) {
+// Lane 0's part of committing a fully copied running request `sl` of source s
+// to its destination (Sec. 3.5, Fig. 4).  The warp has already taken the
+// slot out of s's running list (order kept); fm is the new minimum finishing
+// formation of what is left there.
+__device__ __forceinline__ void commit_book(const Ctx &x, Cnt &cn, int s, const uint4 &sl, uint32_t fm) {
     const int d = x.mpeer[s];
-    const uint4 sl = *slot_ptr(x, s, pos);
     const int blocks = sl_blocks(x, s, sl);
     const uint32_t adv = sl_adv(x, s, sl);
-    slot_remove(x, s, pos);
-    if (sl_fin(sl) == x.minfin[s]) recompute_minfin(x, s);
+    x.nrun[s] = (uint8_t)(x.nrun[s] - 1);
+    x.hist[s * x.TH + sl_rho(sl)]--;
+    x.minfin[s] = fm;
     x.free_[s] += blocks;
     x.resv[d] -= x.mcopied[s];
     const uint32_t tr = sl_tier(sl);
@@ -490,15 +464,29 @@ __device__ __forceinline__ void coop_stage(const Ctx &x, Cnt &cn, int s) {
     commit = __shfl_sync(kFull, commit, 0);
     __syncwarp();
     if (commit) {
+        // the whole warp finds the request's slot (lane l holds slots l and
+        // 32 + l), closes the gap and takes the survivors' minimum; lane 0 books
         const uint32_t rid = x.mreq[s];
         const int n = x.nrun[s];
-        const uint4 *p = slot_ptr(x, s, 0);
-        const uint32_t h0 = __ballot_sync(kFull, x.lane < n && p[x.lane].x == rid);
-        const uint32_t h1 = __ballot_sync(kFull, x.lane + 32 < n && p[x.lane + 32].x == rid);
+        uint4 *p = slot_ptr(x, s, 0);
+        const int q0 = x.lane, q1 = x.lane + 32;
+        const bool v0 = q0 < n, v1 = q1 < n;
+        const uint4 a0 = v0 ? p[q0] : make_uint4(0, 0, 0, 0);
+        const uint4 a1 = v1 ? p[q1] : make_uint4(0, 0, 0, 0);
+        const uint32_t h0 = __ballot_sync(kFull, v0 && a0.x == rid);
+        const uint32_t h1 = __ballot_sync(kFull, v1 && a1.x == rid);
         const int pos = h0 ? __ffs(h0) - 1 : (h1 ? 32 + __ffs(h1) - 1 : -1);
-        if (x.lane == 0) {
-            if (pos < 0) cn.status = SIM_ERR_INTERNAL;
-            else commit_mig(x, cn, s, pos);
+        if (pos < 0) {
+            if (x.lane == 0) cn.status = SIM_ERR_INTERNAL;
+        } else {
+            const uint4 sl = p[pos];
+            const uint32_t fm = __reduce_min_sync(
+                kFull, min(v0 && q0 != pos ? sl_fin(a0) : kNone, v1 && q1 != pos ? sl_fin(a1) : kNone));
+            __syncwarp();
+            if (v0 && q0 > pos) p[q0 - 1] = a0;
+            if (v1 && q1 > pos) p[q1 - 1] = a1;
+            __syncwarp();
+            if (x.lane == 0) commit_book(x, cn, s, sl, fm);
         }
         __syncwarp();
     }
@@ -611,24 +599,37 @@ __device__ __forceinline__ void inst_form(const Ctx &x, Cnt &cn, int i, int base
             need = x.hol[i];
         }
     }
-    // (ii) admission
+    // (ii) admission; the waiting mask and the HoL demand follow in registers
     const int n_decode = n;
     int prefill = 0;
     while (n < x.Bmax) {
         if (!wm) break;
         if (need > fr) break;
         const int k = __ffs(wm) - 1;
-        const uint32_t info = x.hinfo[i * x.K + k];
-        const uint32_t r = pop_front(x, i, k, cn.status);
-        if (r == kNone) break;
+        const int b = i * x.K + k;
+        const uint32_t info = x.hinfo[b];
+        const uint32_t r = x.head[b];
+        if (r >= x.Q) { cn.status = SIM_ERR_INTERNAL; break; }
+        const uint4 nd = x.node[r];  // the head leaves its bucket; nd.x is the new head
+        x.head[b] = nd.x;
         const uint32_t c = info & 0xFFFFu;
         slot_join_at(x, i, n, r, c, info >> 16, (uint32_t)k, nf, ph);
         ++n;
         fr -= need;
         prefill += (int)c;
-        refresh_hol(x, i);
-        wm = x.wmask[i];
-        need = x.hol[i];
+        uint32_t hinfo;  // info of the new head of line
+        if (nd.x != kNone) {
+            x.node[nd.x].z = kNone;
+            x.hinfo[b] = nd.y;
+            hinfo = nd.y;
+        } else {
+            x.tail[b] = kNone;
+            wm &= ~(1u << k);
+            x.wmask[i] = (uint16_t)wm;
+            hinfo = wm ? x.hinfo[i * x.K + (__ffs(wm) - 1)] : 0u;
+        }
+        need = wm ? blocks_for(x, hinfo & 0xFFFFu) : 0;
+        x.hol[i] = need;
     }
     x.nrun[i] = (uint8_t)n;
     x.free_[i] = fr;
