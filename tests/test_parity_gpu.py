@@ -210,3 +210,35 @@ def test_workload1_full_size_sampled():
     ref = parity.run_oracle(w, reps, event_log_capacity=1 << 14)
     for r in reps:
         parity.compare_replica(w, r, res, st, events, ref[r])
+
+
+def test_workload2_full_size_sampled():
+    """The 3,840-replica sweep at full size: sampled replicas (K = 1, 5 and
+    10, each tier distribution, both loads) bit-exact, properties for all."""
+    w = W.config(2)
+    res, st, events = parity.run_gpu(w, event_log_capacity=1 << 14)
+    parity.check_properties(w, res, st)
+    reps = [((k * 3 + d) * 2 + ld) * 64 + 17 * k % 64 for k in (0, 4, 9) for d in range(3) for ld in range(2)]
+    ref = parity.run_oracle(w, reps, event_log_capacity=1 << 14)
+    for r in reps:
+        parity.compare_replica(w, r, res, st, events, ref[r])
+
+
+def test_workload3_full_size_sampled():
+    """The 256-replica, 128-instance bursty workload at full size (200,000
+    requests per replica): first, middle and last replica bit-exact,
+    properties for all."""
+    w = W.config(3)
+    res, st, events = parity.run_gpu(w, event_log_capacity=1 << 14)
+    parity.check_properties(w, res, st)
+    reps = [0, 128, 255]
+    ref = parity.run_oracle(w, reps, event_log_capacity=1 << 14)
+    for r in reps:
+        parity.compare_replica(w, r, res, st, events, ref[r])
+
+
+def test_workload4_full_requests_sample():
+    """Replicas of the 16,384-replica workload with their full 50,000-request
+    traces, bit-exact."""
+    w = W.config(4, replicas=[0, 8191, 16383])
+    parity.check_parity(w, event_log_capacity=1 << 14)
