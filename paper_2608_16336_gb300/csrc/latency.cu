@@ -28,45 +28,51 @@ __device__ __forceinline__ uint32_t lat_floor(uint32_t b) {
 
 // Per-tier latency histograms, sums and maxima.  The requests are cut into
 // chunks of at most kChunk within one replica (chunk_rep / chunk_b0); a
-// block streams one chunk (grid-stride over chunks), histograms it in shared
-// memory while every lane keeps its own exact sums and maxima per (tier,
-// measure) in registers (KM >= the number of tiers, a compile-time bound so
-// the accumulators stay in registers), and merges them into out[r] with
-// global atomics (non-empty buckets only).  out must be zero on entry.
+// block streams one chunk (grid-stride over chunks).  Shared memory holds the
+// chunk's histogram [G][SIM_HIST_BUCKETS] and, per thread, an exact sum and a
+// maximum for every (tier, measure) group, [G][blockDim.x] each, so a request
+// updates only its own group: one histogram atomic, one 64-bit add and one
+// maximum per measure.  At the end of the chunk each warp folds the threads'
+// sums and maxima of some groups and the block merges everything into out[r]
+// with global atomics (non-empty buckets only).  out must be zero on entry.
 // Measures: TTFT = first - arrival, TBT = floor((finish - first) / (O - 1))
 // for O >= 2, E2E = finish - arrival, over finished requests.
-template <int KM>
-__global__ void __launch_bounds__(256) k_latency_hist(const int *chunk_rep, const long long *chunk_b0, int nchunks,
-                                                      const long long *offsets, int KT, const uint32_t *arrival,
-                                                      const uint16_t *olen, const uint8_t *tier,
-                                                      const sim_request_result_t *res, sim_latency_stats_t *out) {
+__global__ void k_latency_hist(const int *chunk_rep, const long long *chunk_b0, int nchunks,
+                               const long long *offsets, int KT, const uint32_t *arrival, const uint16_t *olen,
+                               const uint8_t *tier, const sim_request_result_t *res, sim_latency_stats_t *out) {
     extern __shared__ __align__(16) unsigned char lsm[];
-    const int G = KT * 3;                                  // groups (tier, measure)
-    uint32_t *hist = reinterpret_cast<uint32_t *>(lsm);    // [G][SIM_HIST_BUCKETS]
-    const int lane = threadIdx.x & 31;
+    const int G = KT * 3;  // groups (tier, measure)
+    const int B = (int)blockDim.x;
+    unsigned long long *ssum = reinterpret_cast<unsigned long long *>(lsm);  // [G][B]
+    uint32_t *smax = reinterpret_cast<uint32_t *>(ssum + (size_t)G * B);      // [G][B]
+    uint32_t *hist = smax + (size_t)G * B;                                    // [G][SIM_HIST_BUCKETS]
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = B >> 5;
     for (int c = blockIdx.x; c < nchunks; c += gridDim.x) {
         const int r = chunk_rep[c];
-        const long long b0 = chunk_b0[c], b1 = min(b0 + (long long)kChunk, offsets[r + 1]);
-        for (int q = threadIdx.x; q < G * SIM_HIST_BUCKETS; q += blockDim.x) hist[q] = 0;
-        unsigned long long acc[KM][3];
-        uint32_t amx[KM][3];
-#pragma unroll
-        for (int kk = 0; kk < KM; ++kk)
-#pragma unroll
-            for (int m = 0; m < 3; ++m) { acc[kk][m] = 0; amx[kk][m] = 0; }
+        const long long b0 = chunk_b0[c];
+        const uint32_t nrec = (uint32_t)(min(b0 + (long long)kChunk, offsets[r + 1]) - b0);
+        for (int q = threadIdx.x; q < G * SIM_HIST_BUCKETS; q += B) hist[q] = 0;
+        for (int g = 0; g < G; ++g) {
+            ssum[g * B + threadIdx.x] = 0;
+            smax[g * B + threadIdx.x] = 0;
+        }
         __syncthreads();
+        const uint4 *rs = reinterpret_cast<const uint4 *>(res + b0);
+        const uint32_t *ar = arrival + b0;
+        const uint16_t *ol = olen + b0;
+        const uint8_t *tr = tier + b0;
         constexpr int U = 4;  // requests per thread per pass: their loads are issued together
-        for (long long base = b0 + threadIdx.x; base < b1; base += (long long)U * blockDim.x) {
+        for (uint32_t q0 = threadIdx.x; q0 < nrec; q0 += (uint32_t)(U * B)) {
             uint4 rv[U];
             uint32_t a[U], o[U], k[U];
 #pragma unroll
             for (int u = 0; u < U; ++u) {
-                const long long i = base + (long long)u * blockDim.x;
-                const bool in = i < b1;
-                rv[u] = in ? reinterpret_cast<const uint4 *>(res)[i] : make_uint4(0, 0, kNone, 0);
-                a[u] = in ? arrival[i] : 0u;
-                o[u] = in ? (uint32_t)olen[i] : 0u;
-                k[u] = in ? (uint32_t)tier[i] : 0u;
+                const uint32_t q = q0 + (uint32_t)(u * B);
+                const bool in = q < nrec;
+                rv[u] = in ? rs[q] : make_uint4(0, 0, kNone, 0);
+                a[u] = in ? ar[q] : 0u;
+                o[u] = in ? (uint32_t)ol[q] : 0u;
+                k[u] = in ? (uint32_t)tr[q] : 0u;
             }
 #pragma unroll
             for (int u = 0; u < U; ++u) {
@@ -78,39 +84,33 @@ __global__ void __launch_bounds__(256) k_latency_hist(const int *chunk_rep, cons
                 v[1] = has_tbt ? (fin - first) / (o[u] - 1u) : 0u;
                 v[2] = fin - a[u];
 #pragma unroll
-                for (int m = 0; m < 3; ++m)
-                    if (m != 1 || has_tbt) atomicAdd(&hist[(k[u] * 3 + m) * SIM_HIST_BUCKETS + lat_bucket(v[m])], 1u);
-                // every accumulator is updated with a select (never indexed by the
-                // tier), so all of them stay in registers; a one-token request's
-                // TBT is 0: it adds nothing and leaves the maximum
-#pragma unroll
-                for (int kk = 0; kk < KM; ++kk) {
-                    const bool hit = k[u] == (uint32_t)kk;
-#pragma unroll
-                    for (int m = 0; m < 3; ++m) {
-                        acc[kk][m] += hit ? (unsigned long long)v[m] : 0ull;
-                        amx[kk][m] = hit ? max(amx[kk][m], v[m]) : amx[kk][m];
-                    }
+                for (int m = 0; m < 3; ++m) {
+                    if (m == 1 && !has_tbt) continue;  // a one-token request has no TBT
+                    const int g = (int)k[u] * 3 + m;
+                    atomicAdd(&hist[g * SIM_HIST_BUCKETS + lat_bucket(v[m])], 1u);
+                    const int at = g * B + (int)threadIdx.x;
+                    ssum[at] += v[m];
+                    smax[at] = max(smax[at], v[m]);
                 }
             }
         }
-        // the lanes' sums and maxima: warp reduction, one global atomic per warp and group
-        sim_latency_stats_t *orow = out + (size_t)r * G;
-#pragma unroll
-        for (int kk = 0; kk < KM; ++kk) {
-#pragma unroll
-            for (int m = 0; m < 3; ++m) {
-                if (kk >= KT) continue;  // warp-uniform
-                unsigned long long sv = acc[kk][m];
-#pragma unroll
-                for (int sh = 16; sh > 0; sh >>= 1) sv += __shfl_xor_sync(kFull, sv, sh);
-                const uint32_t mv = __reduce_max_sync(kFull, amx[kk][m]);
-                if (lane == 0 && sv) atomicAdd(reinterpret_cast<unsigned long long *>(&orow[kk * 3 + m].sum_us), sv);
-                if (lane == 0 && mv) atomicMax(&orow[kk * 3 + m].max_us, mv);
-            }
-        }
         __syncthreads();
-        for (int q = threadIdx.x; q < G * SIM_HIST_BUCKETS; q += blockDim.x) {
+        // the threads' sums and maxima: warp w folds groups w, w + nwarps, ...
+        sim_latency_stats_t *orow = out + (size_t)r * G;
+        for (int g = warp; g < G; g += nwarps) {
+            unsigned long long sv = 0;
+            uint32_t mv = 0;
+            for (int t = lane; t < B; t += 32) {
+                sv += ssum[g * B + t];
+                mv = max(mv, smax[g * B + t]);
+            }
+#pragma unroll
+            for (int sh = 16; sh > 0; sh >>= 1) sv += __shfl_xor_sync(kFull, sv, sh);
+            mv = __reduce_max_sync(kFull, mv);
+            if (lane == 0 && sv) atomicAdd(reinterpret_cast<unsigned long long *>(&orow[g].sum_us), sv);
+            if (lane == 0 && mv) atomicMax(&orow[g].max_us, mv);
+        }
+        for (int q = threadIdx.x; q < G * SIM_HIST_BUCKETS; q += B) {
             const uint32_t h = hist[q];
             if (h) atomicAdd(&orow[q / SIM_HIST_BUCKETS].hist[q % SIM_HIST_BUCKETS], h);
         }
@@ -177,11 +177,17 @@ cudaError_t launch(const int *chunk_rep, const long long *chunk_b0, int nchunks,
     cudaError_t e = cudaMemsetAsync(out, 0, (size_t)ngroups * sizeof(sim_latency_stats_t), stream);
     if (e != cudaSuccess) return e;
     if (nchunks > 0) {
-        const size_t smem = (size_t)KT * 3 * 4 * SIM_HIST_BUCKETS;  // <= 46,080 bytes for K <= 16
+        // threads per block: 256 up to 4 tiers, else 128 (the per-thread
+        // accumulators take 12 bytes per thread and group)
+        const int threads = KT <= 4 ? 256 : 128;
+        const size_t smem = (size_t)KT * 3 * (12u * (size_t)threads + 4u * SIM_HIST_BUCKETS);  // <= 119,808 bytes
+        if (smem > 48 * 1024) {
+            e = cudaFuncSetAttribute(k_latency_hist, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+            if (e != cudaSuccess) return e;
+        }
         const int grid = std::max(1, std::min(nchunks, sms * 16));
-        auto fn = KT <= 2 ? k_latency_hist<2> : KT <= 4 ? k_latency_hist<4> : KT <= 8 ? k_latency_hist<8>
-                                                                                   : k_latency_hist<16>;
-        fn<<<grid, 256, smem, stream>>>(chunk_rep, chunk_b0, nchunks, offsets, KT, arrival, olen, tier, res, out);
+        k_latency_hist<<<grid, threads, smem, stream>>>(chunk_rep, chunk_b0, nchunks, offsets, KT, arrival, olen, tier,
+                                                        res, out);
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }
