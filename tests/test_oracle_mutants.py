@@ -54,6 +54,22 @@ MUTANTS = {
                                          "if (eligible[i] && i != s && (d < 0 || freer(i, d))) d = i;"),
     "drain starts one tick late": ("return c.drain_start_us != nullptr && now >= c.drain_start_us[i];",
                                    "return c.drain_start_us != nullptr && now > c.drain_start_us[i];"),
+    "stage copies every block at once (S ignored)": (
+        "int c_blocks = std::min(c.migrate_blocks_per_iter, r.blocks - s.mig_copied);",
+        "int c_blocks = r.blocks - s.mig_copied;"),
+    "running candidate with the most blocks": ("(a.blocks != b.blocks ? a.blocks < b.blocks : r > best)",
+                                               "(a.blocks != b.blocks ? a.blocks > b.blocks : r > best)"),
+    "arrivals dispatched lowest tier first": ("return req[a].tier < req[b].tier; });",
+                                              "return req[a].tier > req[b].tier; });"),
+    "admission ignores the batch limit": ("while ((int)in.running.size() < c.max_batch) {",
+                                          "while (true) {"),
+    "commit ignores the destination's batch limit": (
+        "if (s.mig_copied == r.blocks && (int)d.running.size() < c.max_batch) commit_migration(si);",
+        "if (s.mig_copied == r.blocks) commit_migration(si);"),
+    "highest-priority preemption victim": ("req[x].tier > req[v].tier ||", "req[x].tier < req[v].tier ||"),
+    "migration gate strict (F_d - F_s > theta)": ("< (int64_t)c.theta_num * dd * ds) break;",
+                                                   "<= (int64_t)c.theta_num * dd * ds) break;"),
+    "admission past a misfit head": ("if (need > in.free_blocks) break;", "if (need > in.free_blocks + need) break;"),
 }
 
 
@@ -62,7 +78,8 @@ def _pins_fail(so_path):
     for check in (lambda: pins.check_tiny_agreement(range(120), so_path=so_path),
                   lambda: _closed_forms(so_path),
                   lambda: apins.check_tiny_drain_agreement(range(200), so_path=so_path),
-                  lambda: _autoscale_closed_form(so_path)):
+                  lambda: _autoscale_closed_form(so_path),
+                  lambda: pins.check_threshold_equality(so_path=so_path)):
         try:
             check()
         except AssertionError:

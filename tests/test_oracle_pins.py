@@ -115,6 +115,28 @@ def test_two_simultaneous_requests_closed_form():
     assert res.stats["steps"] == O2 + 1            # the arrival time plus one per iteration end
 
 
+def check_threshold_equality(so_path=None):
+    """Sec. 3.5 migrates when max F - min F >= theta: equality triggers.  Two
+    instances each run one long request that holds one KV block (T = 64,
+    P = 1), so at the 50 ms tick both have F = (10 - 1) / 1: a difference of
+    exactly 0.  With theta = 0 the tick pairs them (source: least free, lowest
+    index = 0; destination: 1) and starts a staged copy of request 0, which
+    commits at instance 0's next iteration end, 4,020 + 12 * 4,030 us.  With
+    theta = 1/1000 nothing moves at the tick."""
+    tr = (np.array([0, 1], np.uint32), np.array([1, 1], np.uint16), np.array([600, 600], np.uint16),
+          np.array([0, 0], np.uint8))
+    cfg = O.make_config(2, 10, [0], tokens_per_block=64, theta_num=0, theta_den=1, check_invariants=1)
+    ev = O.run_trace(cfg, *tr, so_path=so_path).events()
+    assert ev[:2].tolist() == [[50_000, 0, 0, 1, 1, O.EV_START], [4020 + 12 * 4030, 0, 0, 1, 1, O.EV_COMMIT]]
+    cfg = O.make_config(2, 10, [0], tokens_per_block=64, theta_num=1, theta_den=1000, check_invariants=1)
+    ev = O.run_trace(cfg, *tr, so_path=so_path).events()
+    assert ev.shape[0] == 0 or ev[0, 0] > 50_000
+
+
+def test_migration_threshold_equality():
+    check_threshold_equality()
+
+
 # ----------------------------------------------------------- brute force --
 def _oracle_tiny(n, m, headroom, trace, policy, so_path=None):
     cfg = O.make_config(n, m, headroom, check_invariants=1, **policy)
