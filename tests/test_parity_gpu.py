@@ -199,6 +199,17 @@ def test_malformed_trace_rejected():
         sim.close()
 
 
+def test_migration_threshold_equality():
+    """Freeness difference exactly theta at a tick (theta = 0, equal
+    instances) migrates; theta = 1/1000 does not (Sec. 3.5's >=)."""
+    tr = (np.array([0, 1], np.uint32), np.array([1, 1], np.uint16), np.array([600, 600], np.uint16),
+          np.array([0, 0], np.uint8))
+    for num, den in ((0, 1), (1, 1000)):
+        w = W.custom(2, 10, [1], [[0]], [0, 0], [tr, tr], tokens_per_block=64, theta_num=num, theta_den=den)
+        _, st, _ = parity.check_parity(w)
+        assert (st["migration_starts"] > 0).all() == (num == 0)
+
+
 # ----------------------------------------------------------- full size --
 def test_workload1_full_size_sampled():
     """The 1,024-replica workload at full size, in the launch configuration
