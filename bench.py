@@ -328,10 +328,14 @@ def cpu_baseline(w, nrep: int) -> dict:
     cores = os.cpu_count() or 1
     reps = list(range(min(nrep, w.num_replicas)))
     r = oracle.timed_sample(w, reps, cores)
+    one = oracle.timed_sample(w, reps[:4], 1)  # the same oracle on one core, one replica at a time
     return {"value": r["steps"] / r["seconds"], "unit": UNIT, "cores": cores, "kind": "oracle",
             "sample": "first %d of %d replicas, full 20,000 requests each (%d replica-steps, %.1f s wall)" % (
                 len(reps), w.num_replicas, r["steps"], r["seconds"]),
-            "request_events_per_s": r["events"] / r["seconds"]}
+            "request_events_per_s": r["events"] / r["seconds"],
+            "single_core": {"value": one["steps"] / one["seconds"], "unit": UNIT,
+                            "sample": "first %d replicas, one after another on one thread (%.2f s)" % (
+                                one["replicas"], one["seconds"])}}
 
 
 def bench_reference(args):
