@@ -1143,12 +1143,18 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, (!SMS && C <= 2) ? 8 : 4)
                 // ---- window [tb, t1): at most one iteration end per instance ----
                 const uint32_t t1 =
                     (uint32_t)min((unsigned long long)tg, (unsigned long long)tb + (uint32_t)p.base);
-                uint32_t cm = 0, solo = 0;  // instances with an iteration end in the window: in a migration / not
+                // instances with an iteration end in the window: stepped with the
+                // others of a migration in time order (cm), or alone (solo).  A
+                // destination whose source has no event in the window is alone:
+                // only the source's events (stages, commit, abort) touch the other end.
+                uint32_t cm = 0, solo = 0;
 #pragma unroll
                 for (int j = 0; j < C; ++j) {
                     const int i = lane * C + j;
                     if (bz[j] < t1) {
-                        if (x.mrole[i] != MIG_NONE) cm |= 1u << j; else solo |= 1u << j;
+                        const int role = x.mrole[i];
+                        if (role == MIG_NONE || (role == MIG_DST && x.busy[x.mpeer[i]] >= t1)) solo |= 1u << j;
+                        else cm |= 1u << j;
                     }
                 }
                 if (C > 1) {
