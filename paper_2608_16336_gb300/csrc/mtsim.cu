@@ -1040,8 +1040,9 @@ __device__ __forceinline__ void form_all(const Ctx &x, Cnt &cn, uint32_t mask, c
 // at least `base` microseconds.  So in a window [tmin, min(T_g, tmin + base))
 // every instance ends at most one iteration, and each lane advances its own
 // instances (an O(1) iteration end + batch formation); instances in a
-// migration, and every step at a global event, are advanced by lane 0 in the
-// oracle's order.  EXT: the variant that also handles draining instances and
+// migration (but a destination whose source has no event in the window), and
+// every step at a global event, are advanced by the warp in the oracle's
+// order.  EXT: the variant that also handles draining instances and
 // the auto-scaling signal (the other variant compiles that code out).
 template <int C, bool SMS, bool EXT>
 // Variants that keep the running-request records in HBM run workloads with
