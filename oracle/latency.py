@@ -11,14 +11,14 @@ end-to-end latency; their means and P50 / P90 / P99):
   (O - 1)), its mean time between tokens; requests with O = 1 have none.
 * Only finished requests count.
 * Percentile p of n values: the nearest-rank value, i.e. the value of rank
-  ceil(p * n / 100) in ascending order (rank 1 when that is 0), reported as
-  the lower bound of its histogram bucket.
+  ceil(p * n / 100) in ascending order (rank 1 when that is 0), exactly (the
+  paper's P50 / P90 / P99 are values of the latency distribution).
 * Histogram buckets of a value v (32-bit): v itself for v < 8; otherwise,
   with e = floor(log2 v), bucket 8 + 8 (e - 3) + (floor(v / 2^(e-3)) - 8),
   i.e. eight equal buckets per power of two.  240 buckets cover every value.
 
-Percentiles here come from sorting the exact values (no histogram), so they
-check the GPU's histogram scan rather than repeat it.
+Percentiles here come from sorting the exact values (no histogram and no
+radix selection), so they check the GPU's selection rather than repeat it.
 """
 from __future__ import annotations
 
@@ -67,14 +67,14 @@ def request_latencies(arrival, output_len, first_token, finish):
 
 
 def tier_stats(values) -> dict:
-    """count, sum, max, histogram and percentile floors of one group."""
+    """count, sum, max, histogram and nearest-rank percentiles of one group."""
     vals = sorted(int(v) for v in values)
     hist = [0] * NUM_BUCKETS
     for v in vals:
         hist[bucket(v)] += 1
     st = {"count": len(vals), "sum": sum(vals), "max": vals[-1] if vals else 0, "hist": hist}
     for p in PERCENTILES:
-        st["p%d" % p] = bucket_floor(bucket(nearest_rank(vals, p))) if vals else 0
+        st["p%d" % p] = nearest_rank(vals, p) if vals else 0
     return st
 
 

@@ -3,7 +3,8 @@
 * The bucket function against its defining properties, by brute force:
   every value lies in [floor(b), floor(b + 1)), buckets are contiguous and
   ordered, eight per power of two, at most 1/8 of their floor wide.
-* Nearest-rank percentiles against numpy's ``inverted_cdf`` percentile.
+* Nearest-rank percentiles against numpy's ``inverted_cdf`` percentile, and
+  the statistics' P50 / P90 / P99 equal to it on the values themselves.
 * Closed forms for a lone request: TTFT = base + a P, TBT = base + b,
   E2E = TTFT + (O - 1)(base + b) under the iteration-time model.
 """
@@ -49,16 +50,25 @@ def test_nearest_rank_matches_numpy(n):
         assert LT.nearest_rank(v, p) == int(np.percentile(v, p, method="inverted_cdf"))
 
 
-def test_percentile_floor_brackets_exact_value():
-    rng = np.random.default_rng(3)
-    v = rng.lognormal(10, 2, size=5000).astype(np.int64)
+@pytest.mark.parametrize("seed,n", [(3, 5000), (4, 1), (5, 2), (6, 7), (7, 101)])
+def test_percentiles_are_exact_values(seed, n):
+    rng = np.random.default_rng(seed)
+    v = rng.lognormal(10, 2, size=n).astype(np.int64)
     st = LT.tier_stats(v)
-    assert sum(st["hist"]) == st["count"] == 5000
+    assert sum(st["hist"]) == st["count"] == n
     assert st["sum"] == int(v.sum()) and st["max"] == int(v.max())
     for p in LT.PERCENTILES:
-        exact = int(np.percentile(v, p, method="inverted_cdf"))
-        f = st["p%d" % p]
-        assert f <= exact and LT.bucket(f) == LT.bucket(exact)
+        assert st["p%d" % p] == int(np.percentile(v, p, method="inverted_cdf"))
+        assert st["p%d" % p] in set(int(x) for x in v)
+
+
+def test_percentiles_with_ties_and_extremes():
+    v = [7] * 50 + [0xFFFFFFFF] * 49 + [0]
+    st = LT.tier_stats(v)
+    assert (st["p50"], st["p90"], st["p99"]) == (7, 0xFFFFFFFF, 0xFFFFFFFF)
+    st = LT.tier_stats([5, 5, 5])
+    assert (st["p50"], st["p90"], st["p99"]) == (5, 5, 5)
+    assert LT.tier_stats([])["p99"] == 0
 
 
 def test_lone_request_closed_forms():
@@ -73,7 +83,7 @@ def test_lone_request_closed_forms():
     assert tbt["sum"] == 4000 + 30
     assert e2e["sum"] == 4000 + 20 * P + (Ob - 1) * (4000 + 30)
     for s in (ttft, tbt, e2e):
-        assert s["p50"] == s["p99"] == LT.bucket_floor(LT.bucket(s["sum"]))
+        assert s["p50"] == s["p90"] == s["p99"] == s["sum"]
     assert all(s["count"] == 0 for s in st[0])
 
 
