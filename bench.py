@@ -1,19 +1,23 @@
 """Throughput of the batched multi-tier scheduler simulation on GB300.
 
-A step is one complete simulation of the benchmark workload -- 1,024
-independent replicas, each a 16-instance x 2,048-block cluster with K = 4
-enterprise-mix tiers and 20,000 requests (Poisson at 0.85 of capacity) -- from
-t = 0 until every request has finished: state reset plus one persistent
-simulation kernel, inputs resident in HBM.  `value` is simulated
-replica-steps per second (a replica-step = one distinct event time processed in
-one replica), summed over GPUs.  `e2e` repeats the measurement through the C
-ABI with the trace in pinned host memory: the host-to-device copy, validation,
-simulation and the device-to-host copy of every per-request result are inside
-the timed region.
+A step is one complete simulation of a workload -- by default the largest
+one, 16,384 independent replicas, each a 64-instance x 2,048-block cluster
+with K = 4 enterprise-mix tiers and 50,000 requests (Poisson at 0.9 of
+capacity) -- from t = 0 until every request has finished: state reset plus one
+persistent simulation kernel, inputs resident in HBM, every migration-log
+record written (the log is sized by a first run so that no replica
+overflows it).  `value` is simulated replica-steps per second (a replica-step
+= one distinct event time processed in one replica), summed over GPUs.  `e2e`
+repeats the measurement through the C ABI with the trace in pinned host
+memory: the host-to-device copy, validation, simulation and the
+device-to-host copy of every per-request result, the per-replica stats and
+the migration log are inside the timed region.  The smaller workloads 0-3 are
+timed after the headline and reported under `other_workloads`.
 
-Multi-GPU (torchrun, one process per GPU): each rank simulates its own
-independent copy of the workload (other seeds); there is no collective on the
-data path, only a barrier and a max/sum of the timings (weak scaling).
+Multi-GPU (torchrun, one process per GPU): the workload's replicas are split
+into contiguous ranges balanced by predicted work (requests x instances x
+load), one range per rank; there is no collective on the data path, only a
+barrier and a max/sum of the timings (total work fixed: strong scaling).
 
 --impl reference times the CPU oracle (the plain single-threaded reference
 simulator, one replica per host thread) on a bounded sample of the same
@@ -22,6 +26,7 @@ workload.
 from __future__ import annotations
 
 import argparse
+import hashlib
 import json
 import os
 import statistics
@@ -36,17 +41,45 @@ if HERE not in sys.path:
 
 import numpy as np  # noqa: E402
 
-WORKLOAD_ID = 1
-WORKLOAD_NAME = ("1,024 replicas x 16 instances x 2,048 KV blocks (16 tokens/block, batch 64), K=4 enterprise tiers "
-                 "(.05/.15/.30/.50), 20,000 requests/replica, Poisson at 0.85 load, H_k = 512 >> k, "
-                 "64 migration blocks/iteration, 50 ms / theta 0.3 rebalancing")
+HEADLINE_WORKLOAD = 4
+WORKLOAD_NAMES = {
+    0: "1 replica x 4 instances x 1,024 KV blocks (16 tokens/block, batch 64), K=2 uniform tiers, 2,000 requests, "
+       "Poisson 8 req/s, H_k = 256 >> k, 64 migration blocks/iteration, 50 ms / theta 0.3 rebalancing",
+    1: "1,024 replicas x 16 instances x 2,048 KV blocks (16 tokens/block, batch 64), K=4 enterprise tiers "
+       "(.05/.15/.30/.50), 20,000 requests/replica, Poisson at 0.85 load, H_k = 512 >> k, "
+       "64 migration blocks/iteration, 50 ms / theta 0.3 rebalancing",
+    2: "3,840-replica sweep (K=1..10 x uniform/gaussian/geometric tiers x load 0.6/0.9 x 64 seeds) x 32 instances "
+       "x 2,048 KV blocks, 10,000 requests/replica, Poisson, H_k = 512 >> k, 64 migration blocks/iteration",
+    3: "256 replicas x 128 instances x 4,096 KV blocks, K=10 gaussian tiers, 200,000 requests/replica, bursty "
+       "Gamma arrivals (CV 3) at 0.95 load, prompts LN(7.0, 1.0) in [16, 8192], H_k = 1024 >> k, "
+       "32 migration blocks/iteration",
+    4: "16,384 replicas x 64 instances x 2,048 KV blocks (16 tokens/block, batch 64), K=4 enterprise tiers "
+       "(.05/.15/.30/.50), 50,000 requests/replica, Poisson at 0.9 load, H_k = 512 >> k, "
+       "64 migration blocks/iteration, 50 ms / theta 0.3 rebalancing",
+}
 METRIC = "simulated replica-steps/sec (1 GB300) and achieved HBM GB/s fraction of peak"
 UNIT = "replica-steps/s"
-# Algorithmic bytes (what the method must move through HBM at minimum):
-BYTES_PER_REQUEST = 9 + 16       # read the trace record, write the result record
+# Algorithmic bytes of the method (the least it must move through HBM):
+BYTES_PER_REQUEST = 9 + 14       # read the trace record (u32, u16, u16, u8), write the result fields
 BYTES_PER_MEMBER_ITERATION = 8   # read + write a running request's 2-byte token and 2-byte block counters
+BYTES_PER_TOUCHED_INSTANCE = 64  # ~32 B of instance state read + written per instance touched in a step
 BYTES_PER_LOG_RECORD = 16        # one migration-log record
 KERNELS_PER_STEP = 3             # k_init_state, k_init_requests, k_run
+
+
+def algorithmic_bytes(q: int, st) -> dict:
+    """Algorithmic bytes of one complete simulation from its exact counters.
+    Touched instance-steps are counted as: each iteration (its end and the
+    next formation touch the instance once), each dispatched request (its
+    destination), and each migration-log record (its source and destination)."""
+    member = float(st["member_iterations"].sum())
+    iters = float(st["iterations"].sum())
+    logs = float(st["log_events"].sum())
+    touched = iters + float(q) + 2.0 * logs
+    total = (q * BYTES_PER_REQUEST + member * BYTES_PER_MEMBER_ITERATION + touched * BYTES_PER_TOUCHED_INSTANCE
+             + logs * BYTES_PER_LOG_RECORD)
+    return {"total": total, "requests": float(q), "member_iterations": member, "iterations": iters,
+            "touched_instance_steps": touched, "log_records": logs}
 
 
 def dist_env():
@@ -87,19 +120,22 @@ def measured_peak_hbm():
         return 6800.0, "fallback"
 
 
-def kernel_traffic(per_launch_units: float):
-    """DRAM bytes per k_run launch from the committed ncu summary, scaled to
-    this launch, or None if the kernel source changed since the capture."""
-    path = os.path.join(HERE, "profiles", "k_run_workload1_traffic.json")
+def kernel_source_hash() -> str:
+    src = os.path.join(HERE, "paper_2608_16336_gb300", "csrc", "mtsim.cu")
+    return hashlib.sha256(open(src, "rb").read()).hexdigest()
+
+
+def profile_record(cid: int):
+    """The committed ncu figures for k_run on (a reduced case of) workload
+    ``cid``: DRAM bytes per request and warp-instructions per replica-step, or
+    None when the kernel source has changed since they were taken."""
+    path = os.path.join(HERE, "profiles", "k_run_workload%d_traffic.json" % cid)
     try:
         with open(path) as f:
             rec = json.load(f)
-        import hashlib
-
-        src = os.path.join(HERE, "paper_2608_16336_gb300", "csrc", "mtsim.cu")
-        if hashlib.sha256(open(src, "rb").read()).hexdigest() != rec["mtsim_cu_sha256"]:
+        if kernel_source_hash() != rec["mtsim_cu_sha256"]:
             return None
-        return float(rec["dram_bytes_per_unit"]) * per_launch_units
+        return rec
     except Exception:
         return None
 
@@ -155,6 +191,61 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
+def sized_simulator(mtsim, w, cap: int, stream):
+    """A simulator whose migration log holds every record of every replica:
+    one complete run with capacity ``cap``; if some replica produced more
+    records, the simulator is rebuilt with exactly enough room.  Returns the
+    simulator (after that run), its capacity and the run's stats."""
+    while True:
+        sim = mtsim.Simulator(w, event_log_capacity=cap, stream=stream)
+        sim.load(on_device=True)
+        mtsim.sim_run(sim.handle, 1 << 62, False)
+        st = sim.stats()
+        need = int(st["log_events"].max()) if len(st) else 0
+        if need <= cap:
+            return sim, cap, st
+        sim.close()
+        sim._trace = None
+        cap = (need + 15) // 16 * 16
+
+
+def initial_log_capacity(w) -> int:
+    q = int(np.diff(w.offsets).max()) if w.num_replicas else 0
+    return max(1024, (q * 3 // 2 + 15) // 16 * 16)
+
+
+def time_device_steps(torch, mtsim, sim, stream, steps: int, warmup: int, clocks=None):
+    """W untimed and K timed complete simulations (reset + run) on the device:
+    (seconds per step over the whole region, mean k_run launch seconds, clocks)."""
+    def step():
+        mtsim.sim_reset(sim.handle)
+        mtsim.sim_run(sim.handle, 1 << 62, False)
+
+    for _ in range(warmup):
+        step()
+    torch.cuda.synchronize()
+    k_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    if clocks:
+        clocks.start()
+    barrier()
+    torch.cuda.synchronize()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for i in range(steps):
+        mtsim.sim_reset(sim.handle)
+        k_ev[i][0].record(stream)
+        mtsim.sim_run(sim.handle, 1 << 62, False)
+        k_ev[i][1].record(stream)
+    t1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    clk = clocks.stop() if clocks else None
+    dev_s = t0.elapsed_time(t1) / 1e3
+    k_s = sum(a.elapsed_time(b) for a, b in k_ev) / 1e3 / steps
+    return dev_s, k_s, clk
+
+
 def bench_gpu(args):
     import torch
 
@@ -168,63 +259,42 @@ def bench_gpu(args):
         torch.cuda.set_device(0)
     from paper_2608_16336_gb300 import mtsim, workloads
 
-    reps = range(args.replicas) if args.replicas else None
-    w = workloads.config(WORKLOAD_ID, replicas=reps, requests=args.requests, seed_block=rank)
+    cid = args.workload
+    r_all = args.replicas or workloads.num_replicas(cid)
+    lo, hi = workloads.partition(workloads.predicted_work(cid, args.requests)[:r_all], ws)[rank]
+    w = workloads.config(cid, replicas=range(lo, hi), requests=args.requests)
     stream = torch.cuda.current_stream()
-    sim = mtsim.Simulator(w, event_log_capacity=args.log_capacity, stream=stream)
-    sim.load(on_device=True)
+    sim, cap, st0 = sized_simulator(mtsim, w, args.log_capacity or initial_log_capacity(w), stream)
     R, Q = w.num_replicas, w.total_requests
 
-    def step():
-        mtsim.sim_reset(sim.handle)
-        mtsim.sim_run(sim.handle, 1 << 62, False)
-
-    for _ in range(args.warmup):
-        step()
-    torch.cuda.synchronize()
-    # per-launch duration of the simulation kernel, on its own stream
-    k_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
     clocks = ClockSampler(local, args.clocks_dir)
-    clocks.start()
-    barrier()
-    torch.cuda.synchronize()
-    t0 = torch.cuda.Event(enable_timing=True)
-    t1 = torch.cuda.Event(enable_timing=True)
-    t0.record(stream)
-    for i in range(args.steps):
-        mtsim.sim_reset(sim.handle)
-        k_ev[i][0].record(stream)
-        mtsim.sim_run(sim.handle, 1 << 62, False)
-        k_ev[i][1].record(stream)
-    t1.record(stream)
-    torch.cuda.synchronize()
-    barrier()
-    clk = clocks.stop()
-    dev_s = t0.elapsed_time(t1) / 1e3
-    k_s = sum(a.elapsed_time(b) for a, b in k_ev) / 1e3 / args.steps
+    dev_s, k_s, clk = time_device_steps(torch, mtsim, sim, stream, args.steps, args.warmup, clocks)
 
-    res, st, _ = sim.metrics()
+    st = sim.stats()
     assert (st["status"] == mtsim.SIM_REPLICA_DONE).all(), "a replica did not finish"
+    assert int(st["log_events"].max()) <= cap, "a replica overflowed its migration log"
+    assert (st["steps"] == st0["steps"]).all() and (st["log_events"] == st0["log_events"]).all()
+    launch = sim.launch_info()
     lat_info = time_latency_stats(torch, mtsim, sim, w, stream)
     steps_per_run = float(st["steps"].sum())
     events_per_run = float(st["events"].sum())
-    member_iters = float(st["member_iterations"].sum())
-    log_recs = float(np.minimum(st["log_events"], args.log_capacity).sum())
-    alg_bytes = Q * BYTES_PER_REQUEST + member_iters * BYTES_PER_MEMBER_ITERATION + log_recs * BYTES_PER_LOG_RECORD
+    alg = algorithmic_bytes(Q, st)
 
-    # end to end through the C ABI with pinned host buffers
+    # end to end through the C ABI with pinned host buffers: trace in, every
+    # result, the per-replica stats and the whole migration log out
     pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
     h_arr, h_p, h_o, h_t = (pin(w.arrival_us.view(np.int32)), pin(w.prompt_len.view(np.int16)),
                             pin(w.output_len.view(np.int16)), pin(w.tier))
     h_res = torch.empty(Q * mtsim.RESULT_DTYPE.itemsize, dtype=torch.uint8).pin_memory()
     h_st = torch.empty(R * mtsim.STATS_DTYPE.itemsize, dtype=torch.uint8).pin_memory()
+    h_ev = torch.empty(R * cap * mtsim.EVENT_DTYPE.itemsize, dtype=torch.uint8).pin_memory()
     off = np.ascontiguousarray(w.offsets, np.int64)
 
     def e2e_step():
         mtsim.sim_load_trace(sim.handle, off.ctypes.data, h_arr.data_ptr(), h_p.data_ptr(), h_o.data_ptr(),
                              h_t.data_ptr(), 0)
         mtsim.sim_run(sim.handle, 1 << 62, False)
-        mtsim.sim_metrics(sim.handle, h_res.data_ptr(), h_st.data_ptr(), None, 0)
+        mtsim.sim_metrics(sim.handle, h_res.data_ptr(), h_st.data_ptr(), h_ev.data_ptr(), 0)
 
     e2e_step()
     barrier()
@@ -235,14 +305,32 @@ def bench_gpu(args):
     torch.cuda.synchronize()
     barrier()
     e2e_s = (time.perf_counter() - e0) / args.e2e_steps
+    st_e2e = h_st.numpy().view(mtsim.STATS_DTYPE)
+    assert (st_e2e["steps"] == st["steps"]).all() and (st_e2e["status"] == 0).all()
     h2d = int(off.nbytes + Q * 9)
-    d2h = int(h_res.numel() + h_st.numel())
+    d2h = int(h_res.numel() + h_st.numel() + h_ev.numel())
     sim.close()
+    del sim, h_arr, h_p, h_o, h_t, h_res, h_st, h_ev
 
     tot_s, tot_units, tot_events = aggregate(dev_s, steps_per_run * args.steps, events_per_run * args.steps)
     e2e_max, e2e_units, _ = aggregate(e2e_s, steps_per_run, events_per_run)
     peak, peak_kind = measured_peak_hbm()
-    achieved = alg_bytes / k_s / 1e9
+    achieved = alg["total"] / k_s / 1e9
+    prof = profile_record(cid)
+    sm_mhz = (clk or {}).get("sm_mhz") or 0.0
+    resident = min(R, launch["grid_blocks"] * launch["block_threads"] // 32)
+    latency = {
+        "bound": "dependent instruction chain per replica (one warp per replica)",
+        "sm_mhz": sm_mhz or None,
+        "resident_warps": resident,
+        "replicas": R,
+        "cycles_per_replica_step_per_warp": (k_s * sm_mhz * 1e6 * resident / steps_per_run) if sm_mhz else None,
+        "longest_replica_steps": int(st["steps"].max()),
+        "mean_replica_steps": float(st["steps"].mean()),
+        "cycles_per_step_of_longest_replica": (k_s * sm_mhz * 1e6 / float(st["steps"].max())) if sm_mhz else None,
+        "warp_instructions_per_replica_step": prof.get("warp_instructions_per_replica_step") if prof else None,
+        "launch": launch,
+    }
     line = {
         "metric": METRIC,
         "value": tot_units / tot_s,
@@ -252,17 +340,22 @@ def bench_gpu(args):
         "warmup": args.warmup,
         "ms_per_step": tot_s / args.steps * 1e3,
         "higher_is_better": True,
-        "scaling": "weak",
+        "scaling": "strong",
         "vs_baseline": None,
         "dtype": "int32",
         "data": "synthetic (seeded traces shaped like the paper's workloads; no dataset)",
         "config": {
-            "workload": WORKLOAD_NAME if not (args.replicas or args.requests) else
-            "REDUCED profiling case of: " + WORKLOAD_NAME,
-            "replicas_per_gpu": R,
-            "requests_per_gpu": Q,
+            "workload": WORKLOAD_NAMES[cid] if not (args.replicas or args.requests) else
+            "REDUCED profiling case of: " + WORKLOAD_NAMES[cid],
+            "workload_id": cid,
+            "replicas": r_all,
+            "replicas_this_gpu": [lo, hi],
+            "requests_this_gpu": Q,
             "replica_steps_per_gpu_step": int(steps_per_run),
-            "parallelism": "replicas sharded across GPUs, no collective on the data path",
+            "migration_log_capacity": cap,
+            "migration_log_records": int(st["log_events"].sum()),
+            "max_log_records_per_replica": int(st["log_events"].max()),
+            "parallelism": "replicas partitioned across GPUs by predicted work, no collective on the data path",
             "l2": "inputs larger than L2: trace %.0f MB + per-request state %.0f MB resident" % (
                 Q * 9 / 1e6, Q * 32 / 1e6),
         },
@@ -276,22 +369,46 @@ def bench_gpu(args):
             "peak_kind": peak_kind,
             "unit": "GB/s",
             "frac": achieved / peak,
-            "traffic": kernel_traffic(Q),
+            "traffic": float(prof["dram_bytes_per_request"]) * Q if prof else None,
             "kernel": "k_run",
             "kernel_ms": k_s * 1e3,
-            "algorithmic_bytes_per_launch": alg_bytes,
+            "algorithmic_bytes_per_launch": alg["total"],
+            "algorithmic_terms": alg,
         },
+        "latency": latency,
         "clocks": clk,
         "aux_kernels": [lat_info],
     }
+    if ws == 1 and not args.no_others:
+        line["other_workloads"] = [bench_other(torch, mtsim, workloads, c, stream, args)
+                                   for c in sorted(WORKLOAD_NAMES) if c != cid]
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(w, args.cpu_replicas)
+        line["cpu_baseline"] = cpu_baseline(w, cid, args.cpu_replicas)
     if rank == 0:
         print(json.dumps(line), flush=True)
     if ws > 1:
         import torch.distributed as dist
 
         dist.destroy_process_group()
+
+
+def bench_other(torch, mtsim, workloads, cid: int, stream, args) -> dict:
+    """One smaller workload at full size, timed the same way (3 warm-up and
+    3 timed complete simulations, every log record kept)."""
+    w = workloads.config(cid)
+    sim, cap, _ = sized_simulator(mtsim, w, initial_log_capacity(w), stream)
+    dev_s, k_s, _ = time_device_steps(torch, mtsim, sim, stream, 3, 3)
+    st = sim.stats()
+    launch = sim.launch_info()
+    sim.close()
+    assert (st["status"] == mtsim.SIM_REPLICA_DONE).all() and int(st["log_events"].max()) <= cap
+    alg = algorithmic_bytes(w.total_requests, st)
+    peak, _ = measured_peak_hbm()
+    steps = float(st["steps"].sum())
+    return {"workload_id": cid, "workload": WORKLOAD_NAMES[cid], "value": steps / (dev_s / 3), "unit": UNIT,
+            "ms_per_step": dev_s / 3 * 1e3, "kernel_ms": k_s * 1e3, "replica_steps": int(steps),
+            "longest_replica_steps": int(st["steps"].max()), "migration_log_capacity": cap,
+            "hbm_frac": alg["total"] / k_s / 1e9 / peak, "launch": launch}
 
 
 def time_latency_stats(torch, mtsim, sim, w, stream, reps: int = 10) -> dict:
@@ -320,18 +437,19 @@ def time_latency_stats(torch, mtsim, sim, w, stream, reps: int = 10) -> dict:
             "peak_kind": kind, "unit": "GB/s", "frac": gbs / peak}
 
 
-def cpu_baseline(w, nrep: int) -> dict:
-    """The oracle, as it stands, on the first `nrep` replicas of the same workload,
-    one replica per host thread on all host cores."""
+def cpu_baseline(w, cid: int, nrep: int) -> dict:
+    """The oracle, as it stands, on the first `nrep` replicas of the same
+    workload, one replica per host thread on all host cores."""
     from oracle import oracle
 
     cores = os.cpu_count() or 1
     reps = list(range(min(nrep, w.num_replicas)))
+    q = int(np.diff(w.offsets).max())
     r = oracle.timed_sample(w, reps, cores)
     one = oracle.timed_sample(w, reps[:4], 1)  # the same oracle on one core, one replica at a time
     return {"value": r["steps"] / r["seconds"], "unit": UNIT, "cores": cores, "kind": "oracle",
-            "sample": "first %d of %d replicas, full 20,000 requests each (%d replica-steps, %.1f s wall)" % (
-                len(reps), w.num_replicas, r["steps"], r["seconds"]),
+            "sample": "first %d of %d replicas of workload %d, full %d requests each (%d replica-steps, %.1f s wall)"
+                      % (len(reps), w.num_replicas, cid, q, r["steps"], r["seconds"]),
             "request_events_per_s": r["events"] / r["seconds"],
             "single_core": {"value": one["steps"] / one["seconds"], "unit": UNIT,
                             "sample": "first %d replicas, one after another on one thread (%.2f s)" % (
@@ -345,11 +463,13 @@ def bench_reference(args):
     from oracle import oracle
     from paper_2608_16336_gb300 import workloads
 
-    w = workloads.config(WORKLOAD_ID)
+    cid = args.workload
     cores = os.cpu_count() or 1
-    reps = list(range(min(args.cpu_replicas_per_step, w.num_replicas)))
+    n = min(args.cpu_replicas_per_step, workloads.num_replicas(cid))
+    w = workloads.config(cid, replicas=range(n))
+    reps = list(range(n))
     for _ in range(args.warmup):
-        oracle.timed_sample(w, reps[: max(1, cores)], cores)
+        oracle.timed_sample(w, reps[: max(1, min(cores, n))], cores)
     tot_s, tot_steps, tot_events = 0.0, 0, 0
     for i in range(args.steps):
         r = oracle.timed_sample(w, reps, cores)
@@ -357,6 +477,8 @@ def bench_reference(args):
         tot_steps += r["steps"]
         tot_events += r["events"]
     value = tot_steps / tot_s
+    sample = "first %d of %d replicas of workload %d per step, full requests" % (
+        n, workloads.num_replicas(cid), cid)
     line = {
         "impl": "reference",
         "metric": METRIC,
@@ -367,15 +489,13 @@ def bench_reference(args):
         "warmup": args.warmup,
         "ms_per_step": tot_s / args.steps * 1e3,
         "higher_is_better": True,
-        "scaling": "weak",
+        "scaling": "strong",
         "vs_baseline": None,
         "dtype": "int64",
         "data": "synthetic (seeded traces shaped like the paper's workloads; no dataset)",
-        "config": {"workload": WORKLOAD_NAME,
-                   "sample_per_step": "first %d of 1,024 replicas, full requests" % len(reps)},
+        "config": {"workload": WORKLOAD_NAMES[cid], "workload_id": cid, "sample_per_step": sample},
         "request_events_per_s": tot_events / tot_s,
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
-                         "sample": "first %d of 1,024 replicas per step" % len(reps)},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -387,11 +507,14 @@ def main():
     ap.add_argument("--steps", type=int, default=5)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
+    ap.add_argument("--workload", type=int, default=HEADLINE_WORKLOAD, choices=sorted(WORKLOAD_NAMES))
     ap.add_argument("--e2e-steps", type=int, default=2)
-    ap.add_argument("--log-capacity", type=int, default=4096)
-    ap.add_argument("--cpu-replicas", type=int, default=256)
+    ap.add_argument("--log-capacity", type=int, default=0,
+                    help="initial migration-log capacity per replica (0: 1.5 x requests); grown to fit every record")
+    ap.add_argument("--cpu-replicas", type=int, default=192)
     ap.add_argument("--cpu-replicas-per-step", type=int, default=64)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-others", action="store_true", help="skip the smaller workloads' lines")
     ap.add_argument("--clocks-dir", default=os.path.join(tempfile.gettempdir(), "mtsim_bench"),
                     help="where the raw nvidia-smi clock samples of the timed region are written")
     ap.add_argument("--replicas", type=int, default=0, help="profiling only: first N replicas of the workload")

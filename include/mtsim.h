@@ -69,6 +69,7 @@ extern "C" {
 #define SIM_ERR_CUDA (-7)       /* CUDA runtime error; the object should be destroyed */
 #define SIM_ERR_INTERNAL (-8)   /* a device-side consistency check failed */
 #define SIM_ERR_DEADLOCK (-10)  /* no event left while requests are unfinished */
+#define SIM_ERR_UNFINISHED (-11) /* sim_run_static: some replica did not reach SIM_REPLICA_DONE */
 
 /* Per-replica status (sim_replica_stats_t.status). */
 #define SIM_REPLICA_DONE 0      /* every request of the replica has finished */
@@ -293,6 +294,26 @@ const char *sim_strerror(int code);
 /* Device bytes the object holds (0 for NULL). */
 size_t sim_device_bytes(const sim_t *sim);
 
+/* Launch configuration of the simulation kernel that the next sim_run on
+ * this object will use (a measurement aid: with it, kernel time, SM clock and
+ * step counts give cycles per replica-step per resident warp).  The paper has
+ * no counterpart.  One warp simulates one replica; the grid is persistent
+ * and takes replicas from a work counter. */
+typedef struct {
+    int32_t grid_blocks;        /* blocks of one sim_run launch */
+    int32_t block_threads;      /* threads per block (32 per replica in flight) */
+    int32_t blocks_per_sm;      /* resident blocks per SM that registers and shared memory allow */
+    int32_t instances_per_lane; /* instances each lane of a replica's warp owns */
+    int32_t slots_in_shared;    /* 1: running-request records stay in shared memory while a warp owns a replica */
+    int32_t extended;           /* 1: the variant with draining and the auto-scaling signal */
+    int64_t shared_bytes;       /* dynamic shared memory per block */
+} sim_launch_info_t;
+
+/* Fills *out (host) for the kernel variant sim_run would launch now (it
+ * depends on whether a drain schedule is set or the auto-scaling signal is
+ * on).  Returns SIM_ERR_ARG for NULL arguments. */
+int sim_launch_info(const sim_t *sim, sim_launch_info_t *out);
+
 /* Scratch memory behind sim_run_static: one fixed device array per GPU. */
 #define SIM_STATIC_SCRATCH_BYTES (32u << 20)
 
@@ -317,14 +338,19 @@ size_t sim_device_bytes(const sim_t *sim);
  *
  * Limits: the state of all replicas must fit in the scratch array, about
  * R * (N * (67 + 14 * K + T) + N * Bmax * 16 + 600) + 16 * total records bytes;
- * a larger problem returns SIM_ERR_ARG with the size it needed.  The first
- * call on a device looks up the array's device address (cudaGetSymbolAddress)
- * with that device current, so make the first call before any stream capture.
+ * a larger problem returns SIM_ERR_ARG with the size it needed.  Every call
+ * looks up the array's device address (cudaGetSymbolAddress) with the
+ * caller's device current, so the address stays right after a
+ * cudaDeviceReset; the first call on a device also loads the library's
+ * kernels there, so make the first call before any stream capture.
  * Every call uses the same array and overwrites what the previous call left
  * there; two calls whose work overlaps on the GPU (other streams, other host
  * threads) race and corrupt each other's results.  Validates the trace
- * (SIM_ERR_TRACE) and synchronises the stream before returning.  Errors are
- * described by sim_last_error(NULL). */
+ * (SIM_ERR_TRACE) and synchronises the stream before returning.  Returns
+ * SIM_ERR_UNFINISHED, with every output written, when some replica did not
+ * finish: per_replica[r].status then gives each replica's outcome (a
+ * negative SIM_ERR_* code, or SIM_REPLICA_RUNNING if it reached 2^32 - 1
+ * steps).  Errors are described by sim_last_error(NULL). */
 int sim_run_static(const sim_cluster_t *cluster, const sim_tier_table_t *tiers, const sim_policy_t *policy,
                    const int64_t *replica_offsets, const uint32_t *arrival_us, const uint16_t *prompt_len,
                    const uint16_t *output_len, const uint8_t *tier, sim_request_result_t *per_request,

@@ -1439,6 +1439,9 @@ RunKernel pick(int c) {  // c = instances per lane
 struct Launch {
     RunKernel fn = nullptr, fn_ext = nullptr;
     int grid = 0, grid_ext = 0;
+    int per_sm = 0, per_sm_ext = 0;  // resident blocks per SM of each variant
+    int c = 1;                       // instances per lane
+    bool sms = false;                // running-request records in shared memory
     size_t smem = 0;
 };
 
@@ -1493,6 +1496,8 @@ constexpr uint32_t kSmemSlotLimit = 24u * 1024u;
 inline cudaError_t plan_launch(int R, int N, int Bmax, const Layout &L, Launch &out) {
     const uint32_t slot_bytes = (uint32_t)N * (uint32_t)Bmax * 16u;
     const bool sms = slot_bytes <= kSmemSlotLimit;
+    out.c = lanes_c(N);
+    out.sms = sms;
     out.fn = sms ? pick<true, false>(lanes_c(N)) : pick<false, false>(lanes_c(N));
     out.fn_ext = sms ? pick<true, true>(lanes_c(N)) : pick<false, true>(lanes_c(N));
     out.smem = kMagicBytes + (size_t)kWarpsPerBlock * (L.bytes + (sms ? slot_bytes : 0u) + hash_bytes_for(N));
@@ -1510,6 +1515,7 @@ inline cudaError_t plan_launch(int R, int N, int Bmax, const Layout &L, Launch &
         if (e != cudaSuccess) return e;
         if (per_sm < 1) return cudaErrorInvalidConfiguration;
         (v ? out.grid_ext : out.grid) = (int)std::min<long long>(want, (long long)sms_count * per_sm);
+        (v ? out.per_sm_ext : out.per_sm) = per_sm;
     }
     return e;
 }
@@ -1756,6 +1762,7 @@ const char *sim_strerror(int code) {
         case SIM_ERR_CUDA: return "CUDA runtime error";
         case SIM_ERR_INTERNAL: return "device-side consistency check failed";
         case SIM_ERR_DEADLOCK: return "no pending event while requests are unfinished";
+        case SIM_ERR_UNFINISHED: return "some replica did not finish";
         default: return "unknown error";
     }
 }
@@ -1763,6 +1770,19 @@ const char *sim_strerror(int code) {
 const char *sim_last_error(const sim_t *s) { return s ? s->err.c_str() : g_create_err.c_str(); }
 
 size_t sim_device_bytes(const sim_t *s) { return s ? s->dev_bytes : 0; }
+
+int sim_launch_info(const sim_t *s, sim_launch_info_t *out) {
+    if (!s || !out) return SIM_ERR_ARG;
+    const bool ext = s->d_drain != nullptr || s->pol.autoscale != 0;
+    out->grid_blocks = ext ? s->launch.grid_ext : s->launch.grid;
+    out->block_threads = 32 * mt::kWarpsPerBlock;
+    out->blocks_per_sm = ext ? s->launch.per_sm_ext : s->launch.per_sm;
+    out->instances_per_lane = s->launch.c;
+    out->slots_in_shared = s->launch.sms ? 1 : 0;
+    out->extended = ext ? 1 : 0;
+    out->shared_bytes = (int64_t)s->launch.smem;
+    return SIM_OK;
+}
 
 int sim_create(const sim_cluster_t *cl, const sim_tier_table_t *tt, const sim_policy_t *pol, void *cuda_stream,
                const sim_allocator_t *allocator, sim_t **out) {
@@ -2066,9 +2086,6 @@ static __device__ __align__(256) unsigned char g_static_scratch[SIM_STATIC_SCRAT
 
 namespace {
 
-constexpr int kMaxDevices = 64;
-void *g_static_scratch_addr[kMaxDevices];  // device address of g_static_scratch, looked up once per device
-
 size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 }  // namespace
@@ -2114,15 +2131,14 @@ extern "C" int sim_run_static(const sim_cluster_t *cl, const sim_tier_table_t *t
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return fail(nullptr, SIM_ERR_CUDA, "cudaGetDevice: %s", cudaGetErrorString(e));
-    if (dev < 0 || dev >= kMaxDevices) return fail(nullptr, SIM_ERR_ARG, "device index %d not supported", dev);
-    if (!g_static_scratch_addr[dev]) {
-        void *p = nullptr;
-        e = cudaGetSymbolAddress(&p, g_static_scratch);
-        if (e != cudaSuccess || !p)
-            return fail(nullptr, SIM_ERR_CUDA, "cudaGetSymbolAddress: %s", cudaGetErrorString(e));
-        g_static_scratch_addr[dev] = p;
-    }
-    unsigned char *base = (unsigned char *)g_static_scratch_addr[dev];
+    // The array's device address on the current device, looked up on every
+    // call: a cached address would be stale after a cudaDeviceReset (the
+    // module is loaded again), and nothing shared is written here.
+    void *scratch = nullptr;
+    e = cudaGetSymbolAddress(&scratch, g_static_scratch);
+    if (e != cudaSuccess || !scratch)
+        return fail(nullptr, SIM_ERR_CUDA, "cudaGetSymbolAddress: %s", cudaGetErrorString(e));
+    unsigned char *base = (unsigned char *)scratch;
     cudaStream_t st = (cudaStream_t)cuda_stream;
 
     mt::Launch lc;
@@ -2185,9 +2201,15 @@ extern "C" int sim_run_static(const sim_cluster_t *cl, const sim_tier_table_t *t
         lc.fn<<<lc.grid, 32 * mt::kWarpsPerBlock, lc.smem, st>>>(p);
     uint32_t *ftc = (uint32_t *)(base + o_ftc);
     mt::k_first_tokens<<<std::max(1, std::min(R, sms * 8)), 256, 0, st>>>(p.offsets, R, per_request, ftc);
-    mt::k_export_stats<<<(R + 255) / 256, 256, 0, st>>>(p.rep, per_replica, R, nullptr, ftc);
+    // work[2] (zeroed above) counts the replicas that did not finish
+    mt::k_export_stats<<<(R + 255) / 256, 256, 0, st>>>(p.rep, per_replica, R, p.work + 2, ftc);
+    int unfinished = 0;
     e = cudaGetLastError();
+    if (e == cudaSuccess) e = cudaMemcpyAsync(&unfinished, p.work + 2, 4, cudaMemcpyDeviceToHost, st);
     if (e == cudaSuccess) e = cudaStreamSynchronize(st);
     if (e != cudaSuccess) return fail(nullptr, SIM_ERR_CUDA, "sim_run_static: %s", cudaGetErrorString(e));
+    if (unfinished > 0)
+        return fail(nullptr, SIM_ERR_UNFINISHED, "%d of %d replicas did not finish; see per_replica[r].status",
+                    unfinished, R);
     return SIM_OK;
 }

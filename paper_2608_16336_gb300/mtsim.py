@@ -19,7 +19,7 @@ from . import _build
 
 SIM_OK = 0
 SIM_ERR_ARG, SIM_ERR_TRACE, SIM_ERR_STATE, SIM_ERR_OOM = -1, -2, -3, -4
-SIM_ERR_OVERFLOW, SIM_ERR_CUDA, SIM_ERR_INTERNAL, SIM_ERR_DEADLOCK = -5, -7, -8, -10
+SIM_ERR_OVERFLOW, SIM_ERR_CUDA, SIM_ERR_INTERNAL, SIM_ERR_DEADLOCK, SIM_ERR_UNFINISHED = -5, -7, -8, -10, -11
 SIM_REPLICA_DONE, SIM_REPLICA_RUNNING = 0, 1
 SIM_EV_QUEUED, SIM_EV_START, SIM_EV_COMMIT, SIM_EV_ABORT, SIM_EV_SCALE_OUT, SIM_EV_SCALE_IN = 0, 1, 2, 3, 4, 5
 SIM_NONE32, SIM_NONE16 = 0xFFFFFFFF, 0xFFFF
@@ -64,6 +64,13 @@ class sim_policy_t(ctypes.Structure):
                 ("scale_den", ctypes.c_int32)]
 
 
+class sim_launch_info_t(ctypes.Structure):
+    _fields_ = [("grid_blocks", ctypes.c_int32), ("block_threads", ctypes.c_int32),
+                ("blocks_per_sm", ctypes.c_int32), ("instances_per_lane", ctypes.c_int32),
+                ("slots_in_shared", ctypes.c_int32), ("extended", ctypes.c_int32),
+                ("shared_bytes", ctypes.c_int64)]
+
+
 ALLOC_FN = ctypes.CFUNCTYPE(ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p)
 FREE_FN = ctypes.CFUNCTYPE(None, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p)
 
@@ -74,7 +81,7 @@ class sim_allocator_t(ctypes.Structure):
 
 EXPORTS = ["sim_create", "sim_load_trace", "sim_reset", "sim_run", "sim_metrics", "sim_destroy",
            "sim_last_error", "sim_strerror", "sim_device_bytes", "sim_run_static", "sim_set_drain",
-           "sim_latency_stats"]
+           "sim_latency_stats", "sim_launch_info"]
 SIM_STATIC_SCRATCH_BYTES = 32 << 20
 
 _LIB = None
@@ -114,6 +121,8 @@ def lib() -> ctypes.CDLL:
         L.sim_strerror.restype = ctypes.c_char_p
         L.sim_device_bytes.argtypes = [vp]
         L.sim_device_bytes.restype = ctypes.c_size_t
+        L.sim_launch_info.argtypes = [vp, ctypes.POINTER(sim_launch_info_t)]
+        L.sim_launch_info.restype = ctypes.c_int
         L.sim_run_static.argtypes = [ctypes.POINTER(sim_cluster_t), ctypes.POINTER(sim_tier_table_t),
                                      ctypes.POINTER(sim_policy_t), vp, vp, vp, vp, vp, vp, vp, vp, vp]
         L.sim_run_static.restype = ctypes.c_int
@@ -186,6 +195,13 @@ def sim_destroy(handle) -> None:
 
 def sim_device_bytes(handle) -> int:
     return int(lib().sim_device_bytes(handle))
+
+
+def sim_launch_info(handle) -> dict:
+    """The launch configuration sim_run would use now, as a dict."""
+    out = sim_launch_info_t()
+    _check(lib().sim_launch_info(handle, ctypes.byref(out)), handle)
+    return {name: int(getattr(out, name)) for name, _ in sim_launch_info_t._fields_}
 
 
 def sim_run_static(cluster: sim_cluster_t, tiers: sim_tier_table_t, policy: sim_policy_t, replica_offsets_ptr: int,
@@ -300,6 +316,15 @@ class Simulator:
         sim_metrics(self.handle, res.ctypes.data if len(res) else None, st.ctypes.data,
                     ev.ctypes.data if self.event_log_capacity else None, 0)
         return res, st, ev.reshape(w.num_replicas, -1)[:, : self.event_log_capacity]
+
+    def stats(self) -> np.ndarray:
+        """Per-replica stats only (STATS_DTYPE [R]); nothing else is copied."""
+        st = np.empty(self.w.num_replicas, STATS_DTYPE)
+        sim_metrics(self.handle, None, st.ctypes.data, None, 0)
+        return st
+
+    def launch_info(self) -> dict:
+        return sim_launch_info(self.handle)
 
     def latency_stats(self) -> np.ndarray:
         """Per-tier TTFT / TBT / E2E statistics, LATENCY_DTYPE [R, max tiers, 3]."""

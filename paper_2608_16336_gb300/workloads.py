@@ -289,27 +289,22 @@ CONFIG_NAMES = {
 }
 
 
-def config(cid: int, replicas=None, requests: int | None = None, nthreads: int | None = None,
-           seed_block: int = 0) -> Workload:
-    """Builds workload ``cid`` (0..4).  ``replicas`` selects a subset of replica
-    indices (their seeds are those of the full workload, so a subset is a true
-    sample of it); ``requests`` overrides the per-replica request count;
-    ``seed_block`` > 0 draws an independent copy of the workload (same shapes,
-    other seeds), e.g. one per GPU in a weak-scaling run."""
+def _specs(cid: int):
+    """Shape of workload ``cid``: (N, M, Q, S, per-replica specs, arrival kind, CV).
+    Each spec holds K, the tier distribution, the arrival rate, the load it
+    corresponds to, the length model, H0 and a label."""
     T, BMAX = 16, 64
     if cid == 0:
-        n, m, q = 4, 1024, 2000
-        full = [dict(k=2, dist="uniform", rate=8.0, lens=LEN_DEFAULT, h0=256, label="K2-uniform")]
-        s = 64
-        kind, cv = ARRIVAL_POISSON, 1.0
-        rep_specs = lambda: full
-    elif cid == 1:
+        n, m, q, s = 4, 1024, 2000, 64
+        cap = n * instance_capacity(m, T, BMAX, *_mean_lens(LEN_DEFAULT))
+        specs = [dict(k=2, dist="uniform", rate=8.0, load=8.0 / cap, lens=LEN_DEFAULT, h0=256, label="K2-uniform")]
+        return n, m, q, s, specs, ARRIVAL_POISSON, 1.0
+    if cid == 1:
         n, m, q, s = 16, 2048, 20000, 64
         rate = _load_rate(0.85, n, m, T, BMAX, LEN_DEFAULT)
-        spec = dict(k=4, dist="enterprise", rate=rate, lens=LEN_DEFAULT, h0=512, label="K4-enterprise")
-        rep_specs = lambda: [spec] * 1024
-        kind, cv = ARRIVAL_POISSON, 1.0
-    elif cid == 2:
+        spec = dict(k=4, dist="enterprise", rate=rate, load=0.85, lens=LEN_DEFAULT, h0=512, label="K4-enterprise")
+        return n, m, q, s, [spec] * 1024, ARRIVAL_POISSON, 1.0
+    if cid == 2:
         n, m, q, s = 32, 2048, 10000, 64
         specs = []
         for k in range(1, 11):
@@ -317,25 +312,74 @@ def config(cid: int, replicas=None, requests: int | None = None, nthreads: int |
                 for load in (0.6, 0.9):
                     rate = _load_rate(load, n, m, T, BMAX, LEN_DEFAULT)
                     for _seed in range(64):
-                        specs.append(dict(k=k, dist=dist, rate=rate, lens=LEN_DEFAULT, h0=512,
+                        specs.append(dict(k=k, dist=dist, rate=rate, load=load, lens=LEN_DEFAULT, h0=512,
                                           label="K%d-%s-%.1f" % (k, dist, load)))
-        rep_specs = lambda: specs
-        kind, cv = ARRIVAL_POISSON, 1.0
-    elif cid == 3:
+        return n, m, q, s, specs, ARRIVAL_POISSON, 1.0
+    if cid == 3:
         n, m, q, s = 128, 4096, 200000, 32
         rate = _load_rate(0.95, n, m, T, BMAX, LEN_LONG_PROMPT)
-        spec = dict(k=10, dist="gaussian", rate=rate, lens=LEN_LONG_PROMPT, h0=1024, label="K10-gaussian")
-        rep_specs = lambda: [spec] * 256
-        kind, cv = ARRIVAL_GAMMA, 3.0
-    elif cid == 4:
+        spec = dict(k=10, dist="gaussian", rate=rate, load=0.95, lens=LEN_LONG_PROMPT, h0=1024, label="K10-gaussian")
+        return n, m, q, s, [spec] * 256, ARRIVAL_GAMMA, 3.0
+    if cid == 4:
         n, m, q, s = 64, 2048, 50000, 64
         rate = _load_rate(0.9, n, m, T, BMAX, LEN_DEFAULT)
-        spec = dict(k=4, dist="enterprise", rate=rate, lens=LEN_DEFAULT, h0=512, label="K4-enterprise")
-        rep_specs = lambda: [spec] * 16384
-        kind, cv = ARRIVAL_POISSON, 1.0
-    else:
-        raise ValueError("workload id must be 0..4")
-    specs = rep_specs()
+        spec = dict(k=4, dist="enterprise", rate=rate, load=0.9, lens=LEN_DEFAULT, h0=512, label="K4-enterprise")
+        return n, m, q, s, [spec] * 16384, ARRIVAL_POISSON, 1.0
+    raise ValueError("workload id must be 0..4")
+
+
+def _mean_lens(lens: dict) -> tuple[float, float]:
+    ep = mean_clipped_lognormal(lens["prompt_mu"], lens["prompt_sigma"], lens["prompt_min"], lens["prompt_max"])
+    eo = mean_clipped_lognormal(lens["output_mu"], lens["output_sigma"], lens["output_min"], lens["output_max"])
+    return ep, eo
+
+
+def num_replicas(cid: int) -> int:
+    """Replica count of workload ``cid`` (no trace is generated)."""
+    return len(_specs(cid)[4])
+
+
+def predicted_work(cid: int, requests: int | None = None) -> np.ndarray:
+    """Predicted simulation work of each replica of workload ``cid``,
+    requests x instances x load (float64 [R]); no trace is generated."""
+    n, _m, q, _s, specs, _kind, _cv = _specs(cid)
+    qq = q if requests is None else int(requests)
+    return np.array([float(qq) * n * sp["load"] for sp in specs], dtype=np.float64)
+
+
+def partition(weights, parts: int) -> list[tuple[int, int]]:
+    """Splits replicas 0..R-1 into ``parts`` contiguous ranges [lo, hi) whose
+    summed weights are as even as cutting the prefix sums at multiples of
+    total/parts makes them; every replica lands in exactly one range and every
+    range is non-empty (R >= parts is required)."""
+    w = np.asarray(weights, dtype=np.float64)
+    r = int(w.shape[0])
+    if parts < 1 or r < parts:
+        raise ValueError("need 1 <= parts <= replicas (%d parts, %d replicas)" % (parts, r))
+    if (w < 0).any():
+        raise ValueError("weights must be non-negative")
+    pre = np.concatenate([[0.0], np.cumsum(w)])
+    total = pre[-1]
+    cuts = [0]
+    for k in range(1, parts):
+        c = int(np.searchsorted(pre, total * k / parts, side="left"))
+        # a cut may not leave a range empty, before or after it
+        c = max(c, cuts[-1] + 1)
+        c = min(c, r - (parts - k))
+        cuts.append(c)
+    cuts.append(r)
+    return [(cuts[k], cuts[k + 1]) for k in range(parts)]
+
+
+def config(cid: int, replicas=None, requests: int | None = None, nthreads: int | None = None,
+           seed_block: int = 0) -> Workload:
+    """Builds workload ``cid`` (0..4).  ``replicas`` selects a subset of replica
+    indices (their seeds are those of the full workload, so a subset is a true
+    sample of it); ``requests`` overrides the per-replica request count;
+    ``seed_block`` > 0 draws an independent copy of the workload (same shapes,
+    other seeds)."""
+    T, BMAX = 16, 64
+    n, m, q, s, specs, kind, cv = _specs(cid)
     idx = list(range(len(specs))) if replicas is None else [int(i) for i in replicas]
     if any(i < 0 or i >= len(specs) for i in idx):
         raise ValueError("replica index out of range for workload %d" % cid)

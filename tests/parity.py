@@ -67,16 +67,20 @@ def check_parity(w, replicas=None, **kw):
     return res, st, events
 
 
-def check_properties(w, res, st):
+def check_properties(w, res, st, chunk=1 << 24):
     """Checks that hold for every replica at any size: every request finished
-    once, on a valid instance, no earlier than the iteration-time model allows."""
+    once, on a valid instance, no earlier than the iteration-time model allows.
+    Large traces are checked ``chunk`` records at a time."""
     assert (st["status"] == 0).all()
     assert (st["finished"].astype(np.int64) == np.diff(w.offsets)).all()
-    first = res["first_token_us"].astype(np.int64)
-    fin = res["finish_us"].astype(np.int64)
-    arr = w.arrival_us.astype(np.int64)
-    assert (first != mtsim.SIM_NONE32).all() and (fin != mtsim.SIM_NONE32).all()
-    assert (first - arr >= w.iter_base_us + w.iter_us_per_prefill_token * w.prompt_len.astype(np.int64)).all()
-    assert (fin - first >= (w.output_len.astype(np.int64) - 1) * (w.iter_base_us + w.iter_us_per_decode_seq)).all()
-    assert (res["dispatch_instance"] < w.num_instances).all()
-    assert (res["final_instance"] < w.num_instances).all()
+    for a in range(0, w.total_requests, chunk):
+        b = min(a + chunk, w.total_requests)
+        g = res[a:b]
+        first = g["first_token_us"].astype(np.int64)
+        fin = g["finish_us"].astype(np.int64)
+        arr = w.arrival_us[a:b].astype(np.int64)
+        assert (first != mtsim.SIM_NONE32).all() and (fin != mtsim.SIM_NONE32).all()
+        assert (first - arr >= w.iter_base_us + w.iter_us_per_prefill_token * w.prompt_len[a:b].astype(np.int64)).all()
+        assert (fin - first >= (w.output_len[a:b].astype(np.int64) - 1) * (w.iter_base_us + w.iter_us_per_decode_seq)).all()
+        assert (g["dispatch_instance"] < w.num_instances).all()
+        assert (g["final_instance"] < w.num_instances).all()

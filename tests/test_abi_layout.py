@@ -20,6 +20,7 @@ MIRRORS = {
     "sim_cluster_t": mtsim.sim_cluster_t,
     "sim_tier_table_t": mtsim.sim_tier_table_t,
     "sim_policy_t": mtsim.sim_policy_t,
+    "sim_launch_info_t": mtsim.sim_launch_info_t,
 }
 
 

@@ -24,7 +24,7 @@ def test_reference_line():
     d = json.loads(lines[0])
     assert d["impl"] == "reference" and d["unit"] == "replica-steps/s" and d["higher_is_better"] is True
     assert d["steps"] == 1 and d["warmup"] == 3 and d["n_gpus"] == 1 and d["value"] > 0
-    assert d["config"]["workload"].startswith("1,024 replicas x 16 instances")
+    assert d["config"]["workload"].startswith("16,384 replicas x 64 instances") and d["config"]["workload_id"] == 4
     cb = d["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["value"] == d["value"] and cb["cores"] >= 1 and cb["sample"]
     assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}

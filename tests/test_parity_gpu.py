@@ -4,6 +4,7 @@ migration log and every per-replica counter, on the same seeded inputs."""
 import numpy as np
 import pytest
 
+from paper_2608_16336_gb300 import mtsim
 from paper_2608_16336_gb300 import workloads as W
 from tests import parity
 from tests._tiny import tiny_case
@@ -244,6 +245,32 @@ def test_workload3_full_size_sampled():
     parity.check_properties(w, res, st)
     reps = [0, 128, 255]
     ref = parity.run_oracle(w, reps, event_log_capacity=1 << 14)
+    for r in reps:
+        parity.compare_replica(w, r, res, st, events, ref[r])
+
+
+def test_workload4_full_size_sampled():
+    """The 16,384-replica workload at full size (64 instances, 50,000 requests
+    per replica) in the benchmark's launch: the same kernel variant and grid
+    and a migration log sized, as the benchmark sizes it, to hold every
+    record.  Eight sampled replicas (first, last, spread) bit-exact on every
+    result, every log record and every counter; properties for all."""
+    import bench
+    import torch
+
+    w = W.config(4)
+    sim, cap, st0 = bench.sized_simulator(mtsim, w, bench.initial_log_capacity(w), torch.cuda.current_stream())
+    try:
+        assert sim.launch_info()["instances_per_lane"] == 2 and not sim.launch_info()["slots_in_shared"]
+        res, st, ev = sim.metrics()
+        assert int(st["log_events"].max()) <= cap
+        reps = [0, 1, 2730, 5461, 8191, 10922, 13653, 16383]
+        events = {r: sim.events_of(ev, st, r) for r in reps}
+        del ev
+    finally:
+        sim.close()
+    parity.check_properties(w, res, st)
+    ref = parity.run_oracle(w, reps, event_log_capacity=cap)
     for r in reps:
         parity.compare_replica(w, r, res, st, events, ref[r])
 

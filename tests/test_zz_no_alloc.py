@@ -1,8 +1,9 @@
 """The allocation-free entry point sim_run_static, for callers that cannot
 call cudaMalloc (their device memory belongs to another allocator or budget,
 or they run where an allocation is not allowed).  It must give exactly the
-results of the allocating path (sim_create ... sim_metrics), call after
-call, although every call reuses the same fixed device array."""
+oracle's results and those of the allocating path (sim_create ...
+sim_metrics), call after call, although every call reuses the same fixed
+device array, and a call must not change the device's free memory."""
 import ctypes
 
 import numpy as np
@@ -24,8 +25,9 @@ def torch():
     return t
 
 
-def _static_run(torch, w, cap):
-    """Runs w through sim_run_static with caller-owned device inputs and outputs."""
+def _static_args(torch, w, cap):
+    """sim_run_static's arguments for w: host descriptors, caller-owned device
+    trace and output buffers, the current stream."""
     R = w.num_replicas
     kmax = max(w.tables_k)
     tk = np.asarray(w.tables_k, np.int32)
@@ -45,9 +47,31 @@ def _static_run(torch, w, cap):
     res = torch.empty(w.total_requests * mtsim.RESULT_DTYPE.itemsize, dtype=torch.uint8, device=dev)
     st = torch.empty(R * mtsim.STATS_DTYPE.itemsize, dtype=torch.uint8, device=dev)
     ev = torch.empty(R * cap * mtsim.EVENT_DTYPE.itemsize, dtype=torch.uint8, device=dev)
+    keep = (tk, th, rt, off, tr, res, st, ev)  # the buffers must outlive the call
+    return _StaticArgs(cl, tt, pol, off, tr, res, st, ev, keep)
+
+
+class _StaticArgs(tuple):
+    """(cluster, tiers, policy, offsets ptr, 4 trace ptrs, res ptr, stats ptr,
+    events ptr, stream) plus the tensors behind them."""
+
+    def __new__(cls, cl, tt, pol, off, tr, res, st, ev, keep):
+        import torch as _t
+
+        self = super().__new__(cls, (cl, tt, pol, off.ctypes.data, *[x.data_ptr() for x in tr], res.data_ptr(),
+                                     st.data_ptr(), ev.data_ptr(), _t.cuda.current_stream().cuda_stream))
+        self.keep = keep
+        self.res, self.st, self.ev = res, st, ev
+        return self
+
+
+def _static_run(torch, w, cap):
+    """Runs w through sim_run_static with caller-owned device inputs and outputs."""
+    R = w.num_replicas
+    args = _static_args(torch, w, cap)
+    res, st, ev = args.res, args.st, args.ev
     torch.cuda.synchronize()
-    mtsim.sim_run_static(cl, tt, pol, off.ctypes.data, *[x.data_ptr() for x in tr], res.data_ptr(), st.data_ptr(),
-                         ev.data_ptr(), torch.cuda.current_stream().cuda_stream)
+    mtsim.sim_run_static(*args)
     res_h = res.cpu().numpy().view(mtsim.RESULT_DTYPE)
     st_h = st.cpu().numpy().view(mtsim.STATS_DTYPE)
     ev_h = ev.cpu().numpy().view(mtsim.EVENT_DTYPE).reshape(R, cap)
@@ -64,9 +88,12 @@ def test_static_entry_point_matches_allocating_path(torch):
     cap = 2048
     w = W.config(1, replicas=range(11), requests=2500)
     want = parity.run_gpu(w, event_log_capacity=cap)
+    ref = parity.run_oracle(w, range(w.num_replicas), event_log_capacity=cap)
     for _ in range(2):  # the second call reuses the scratch the first one left behind
         got = _static_run(torch, w, cap)
-        assert (got[0] == want[0]).all()
+        for r in range(w.num_replicas):  # against the oracle itself ...
+            parity.compare_replica(w, r, got[0], got[1], got[2], ref[r])
+        assert (got[0] == want[0]).all()  # ... and the allocating path
         assert (got[1] == want[1]).all()
         for a, b in zip(got[2], want[2]):
             assert (a == b).all()
@@ -75,6 +102,39 @@ def test_static_entry_point_matches_allocating_path(torch):
     want0 = parity.run_gpu(w0, event_log_capacity=cap)
     got0 = _static_run(torch, w0, cap)
     assert (got0[0] == want0[0]).all() and (got0[1] == want0[1]).all()
+
+
+def test_static_entry_point_allocates_nothing(torch):
+    """With the module loaded and the outputs allocated, a call leaves the
+    device's free memory exactly as it found it."""
+    cap = 256
+    w = W.config(0, requests=300)
+    _static_run(torch, w, cap)  # loads the kernels and settles local-memory reservations
+    args = _static_args(torch, w, cap)
+    torch.cuda.synchronize()
+    free0, _ = torch.cuda.mem_get_info()
+    mtsim.sim_run_static(*args)
+    torch.cuda.synchronize()
+    free1, _ = torch.cuda.mem_get_info()
+    assert free1 == free0
+
+
+def test_static_entry_point_reports_unfinished(torch):
+    """A replica that cannot finish (its iteration end overflows 32-bit time)
+    makes the call return SIM_ERR_UNFINISHED, with the replica's status in
+    per_replica."""
+    base = 1 << 24
+    tr = (np.array([0xFFFF0000], np.uint32), np.array([1], np.uint16), np.array([2], np.uint16),
+          np.array([0], np.uint8))
+    ok = (np.array([0], np.uint32), np.array([1], np.uint16), np.array([2], np.uint16), np.array([0], np.uint8))
+    w = W.custom(2, 16, [1], [[0]], [0, 0], [ok, tr], iter_base_us=base)
+    args = _static_args(torch, w, 16)
+    with pytest.raises(mtsim.SimError) as e:
+        mtsim.sim_run_static(*args)
+    assert e.value.code == mtsim.SIM_ERR_UNFINISHED
+    st_h = args.st.cpu().numpy().view(mtsim.STATS_DTYPE)
+    assert int(st_h["status"][0]) == mtsim.SIM_REPLICA_DONE
+    assert int(st_h["status"][1]) == mtsim.SIM_ERR_OVERFLOW
 
 
 def test_static_entry_point_rejects_oversize(torch):
