@@ -5,6 +5,8 @@
 * Closed forms of the iteration-time model for one and two requests.
 * Exact brute force (``tiny_ref``, Fractions) on hundreds of tiny clusters.
 * The K = 2 reduction to the original binary Llumnix headroom (Sec. 3.3).
+* K = 1: the headroom is one constant added whenever the instance holds a
+  request, and with H0 = 0 the schedule is plain freeness-balanced vLLM.
 * Invariants (KV-block conservation, tier isolation, per-tier counts).
 * The paper's qualitative per-tier TTFT ordering (Sec. 5.1).
 """
@@ -188,6 +190,54 @@ def test_tiny_cases_exercise_every_rule():
         pre += int(res.n_preemptions.sum())
     assert kinds == {O.EV_QUEUED, O.EV_START, O.EV_COMMIT, O.EV_ABORT}
     assert pre > 0
+
+
+def test_k1_headroom_is_one_shift_when_present():
+    """K = 1 (Sec. 3.3 Eq. 4 with one tier): U = U(H0 = 0) + H0 when the
+    instance holds any request, U(H0 = 0) when it holds none."""
+    for h0 in (0, 1, 37, 512):
+        cfg, cfg0 = O.make_config(1, 2048, [h0]), O.make_config(1, 2048, [0])
+        for running, hol, cnt in (([], 0, 0), ([], 12, 1), ([5, 9], 0, 2), ([5, 9, 30], 7, 5)):
+            n, d = O.freeness(cfg, running, hol, [cnt])
+            n0, d0 = O.freeness(cfg0, running, hol, [cnt])
+            assert d == d0 == max(len(running), 1)
+            assert n == n0 - (h0 if cnt > 0 else 0)
+            assert n0 == 2048 - sum(running) - hol
+
+
+def test_k1_h0_zero_closed_form_dispatch():
+    """K = 1, H0 = 0 on three empty instances: each arrival goes to the
+    freest instance, lowest index on ties (Sec. 3.4); the fourth finds all
+    three equally loaded and joins instance 0's running prefill's next batch."""
+    P, Ob, T, base, a, b = 160, 50, 16, 4000, 20, 30
+    cfg = O.make_config(3, 2048, [0], tokens_per_block=T, enable_migration=0)
+    res = O.run_trace(cfg, np.array([0, 1, 2, 3], np.uint32), np.full(4, P, np.uint16), np.full(4, Ob, np.uint16),
+                      np.zeros(4, np.uint8))
+    assert list(res.dispatch_instance) == [0, 1, 2, 0]
+    t0 = base + a * P                       # request 0's prefill iteration ends
+    assert int(res.first_token_us[0]) == t0
+    assert int(res.first_token_us[1]) - 1 == t0 and int(res.first_token_us[2]) - 2 == t0
+    # request 3 waited for that iteration, then shares one with request 0's first decode
+    assert int(res.first_token_us[3]) == t0 + base + a * P + b * 1
+
+
+def test_k1_h0_zero_is_plain_freeness_balanced_vllm():
+    """With one tier and no headroom the multi-tier scheduler must give the
+    schedule of the original Llumnix rule with no high-priority headroom,
+    computed by the independent brute force (Fractions): freeness
+    (M - running KV - HoL demand) / B only, FCFS local queues."""
+    for seed in range(150):
+        n, m, _, trace, policy = tiny_case(3000 + seed)
+        trace = (trace[0], trace[1], trace[2], np.zeros_like(trace[3]))
+        res = _oracle_tiny(n, m, [0], trace, policy)
+        sim = _tiny_ref(n, m, [0, 0], (trace[0], trace[1], trace[2], np.ones_like(trace[3])), policy,
+                        binary=True, binary_h=0)
+        _same(res, sim)
+        # and K = 3 with all headroom zero and every request in tier 0 is the same schedule
+        res3 = _oracle_tiny(n, m, [0, 0, 0], trace, policy)
+        assert list(res3.dispatch_instance) == list(res.dispatch_instance)
+        assert list(res3.finish_us) == list(res.finish_us)
+        assert [tuple(e) for e in res3.events().tolist()] == [tuple(e) for e in res.events().tolist()]
 
 
 def test_k2_reduces_to_binary_llumnix():
