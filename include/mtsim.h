@@ -186,9 +186,8 @@ typedef struct {
     uint32_t count;              /* finished requests of the tier counted */
     uint32_t max_us;             /* exact maximum (0 if count = 0) */
     uint64_t sum_us;             /* exact sum; mean = sum_us / count */
-    uint32_t p50_us, p90_us, p99_us; /* nearest-rank percentiles (the value of rank ceil(p * count / 100)),
-                                        rounded down to the floor of their histogram bucket: within
-                                        1/8 below the exact value; 0 if count = 0 */
+    uint32_t p50_us, p90_us, p99_us; /* nearest-rank percentiles: exactly the value of rank
+                                        ceil(p * count / 100) in ascending order; 0 if count = 0 */
     uint32_t pad;
     /* hist[b]: requests whose value v falls in bucket b: b = v for v < 8,
      * else b = 8 * (e - 3) + floor(v / 2^(e-3)) with e = floor(log2 v):
@@ -276,8 +275,9 @@ int sim_metrics(sim_t *sim, sim_request_result_t *per_request, sim_replica_stats
  * requests that have finished, so it may be called between sim_run calls.
  * out is host or device per on_device, [R * max_tiers * 3] records.  Host
  * output synchronises the stream (and allocates a device staging buffer of
- * the same size on first use); device output is asynchronous.  Returns
- * SIM_ERR_STATE before sim_load_trace. */
+ * the same size on first use); device output is asynchronous.  The first
+ * call also allocates the percentile selection scratch, 3,120 bytes per
+ * (replica, tier, measure).  Returns SIM_ERR_STATE before sim_load_trace. */
 int sim_latency_stats(sim_t *sim, sim_latency_stats_t *out, int on_device);
 
 /* Releases everything the object owns (synchronises the stream first).

@@ -1560,6 +1560,8 @@ struct sim {
     sim_latency_stats_t *d_lat = nullptr;  // device staging of sim_latency_stats for host output
     int *d_lat_rep = nullptr;              // chunk table of sim_latency_stats: replica and first record
     long long *d_lat_b0 = nullptr;
+    uint4 *d_lat_sel = nullptr;            // percentile selection scratch of sim_latency_stats
+    uint32_t *d_lat_bins = nullptr;
     int lat_nchunks = -1;                  // -1: to be built for the loaded trace
     int sms = 0;
     std::string err;
@@ -1965,8 +1967,15 @@ int sim_latency_stats(sim_t *s, sim_latency_stats_t *out, int on_device) {
         }
         s->lat_nchunks = nc;
     }
+    if (!s->d_lat_sel) {
+        s->d_lat_sel = (uint4 *)dalloc(s, mtlat::select_state_bytes((long long)n));
+        s->d_lat_bins = (uint32_t *)dalloc(s, mtlat::select_bin_bytes((long long)n));
+        if (!s->d_lat_sel || !s->d_lat_bins)
+            return fail(s, SIM_ERR_OOM, "device allocation of the percentile selection scratch failed");
+    }
     cudaError_t e = mtlat::launch(s->d_lat_rep, s->d_lat_b0, s->lat_nchunks, s->d_off, KT, s->d_arrival, s->d_olen,
-                                  s->d_tier, s->d_res, d, (long long)n, s->sms, s->stream);
+                                  s->d_tier, s->d_res, d, (long long)n, s->d_lat_sel, s->d_lat_bins, s->sms,
+                                  s->stream);
     if (e != cudaSuccess) return cuda_fail(s, e, "sim_latency_stats");
     if (!on_device) {
         e = cudaMemcpyAsync(out, d, n * sizeof(sim_latency_stats_t), cudaMemcpyDeviceToHost, s->stream);

@@ -1,6 +1,6 @@
 """Per-tier latency statistics on the GPU (sim_latency_stats) vs the oracle's
 statistics of the oracle's own results, bit-exact: counts, sums, maxima,
-every histogram bucket and the P50 / P90 / P99 floors."""
+every histogram bucket and the exact P50 / P90 / P99 values."""
 import numpy as np
 import pytest
 
