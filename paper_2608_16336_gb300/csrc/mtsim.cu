@@ -986,6 +986,52 @@ __device__ __forceinline__ void bind_blob(Ctx &x, const Layout &L, unsigned char
     x.mslot = reinterpret_cast<uint4 *>(blob + L.mslot);
 }
 
+// Phase 1 at x.t for the instances in `mask` (bit j = instance lane*C + j)
+// whose iteration ends now, ascending index.  Collective.
+template <int C>
+__device__ __forceinline__ void complete_all(const Ctx &x, Cnt &cn, uint32_t mask) {
+    uint32_t hits = 0;
+#pragma unroll
+    for (int j = 0; j < C; ++j)
+        if (((mask >> j) & 1u) && x.busy[x.lane * C + j] == x.t) hits |= 1u << j;
+    uint32_t lanes = __ballot_sync(kFull, hits != 0);
+    while (lanes) {
+        const int l = __ffs(lanes) - 1;
+        lanes &= lanes - 1;
+        uint32_t h = C == 1 ? 1u : __shfl_sync(kFull, hits, l);
+        while (h) {
+            const int i = l * C + __ffs(h) - 1;
+            h &= h - 1;
+            int fp = 0;
+            if (x.lane == 0) fp = inst_complete_head(x, i);
+            if (__shfl_sync(kFull, fp, 0)) coop_finish(x, cn, i);
+            __syncwarp();
+            if (x.mrole[i] == MIG_SRC) coop_stage(x, cn, i);
+        }
+    }
+}
+
+// Phase 4 at x.t for the idle instances in `mask` that have work, ascending
+// index, on lane 0.  Collective.
+template <int C>
+__device__ __forceinline__ void form_all(const Ctx &x, Cnt &cn, uint32_t mask, const Params &p) {
+    uint32_t want = 0;
+#pragma unroll
+    for (int j = 0; j < C; ++j) {
+        const int i = x.lane * C + j;
+        if (((mask >> j) & 1u) && x.busy[i] == kNone && (x.nrun[i] | x.wmask[i]) != 0) want |= 1u << j;
+    }
+    uint32_t lanes = __ballot_sync(kFull, want != 0);
+    while (lanes) {
+        const int l = __ffs(lanes) - 1;
+        lanes &= lanes - 1;
+        const uint32_t h = C == 1 ? 1u : __shfl_sync(kFull, want, l);
+        if (x.lane == 0)
+            for (uint32_t hh = h; hh; hh &= hh - 1) inst_form(x, cn, l * C + __ffs(hh) - 1, p.base, p.a, p.b);
+    }
+    __syncwarp();
+}
+
 // a[j] for a run-time j without dynamic indexing (the array stays in registers)
 template <int C>
 __device__ __forceinline__ uint32_t pick_c(const uint32_t (&a)[C], int j) {
@@ -995,6 +1041,16 @@ __device__ __forceinline__ uint32_t pick_c(const uint32_t (&a)[C], int j) {
         if (j == k) v = a[k];
     return v;
 }
+
+// Which main loop a variant runs.  The variants that keep running-request
+// records in HBM with at most two instances per lane run 16 warps per SM
+// (many replicas); there instruction fetch was the bottleneck, and a loop
+// in which the window, its migration steps and the global steps share one
+// copy of every phase keeps the hot code small.  The other variants run few
+// warps per SM and are bound by each replica's dependent chain, which the
+// loop with separately inlined phases keeps shorter.
+template <int C, bool SMS>
+constexpr bool kUnifiedLoop = !SMS && C <= 2;
 
 // The persistent simulation kernel: each warp repeatedly takes a replica and
 // advances it by up to p.max_steps event times; C = instances per lane.
@@ -1088,53 +1144,229 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, (!SMS && C <= 2) ? 8 : 4)
         ArrBuf ab;
         arr_refill(x, ab, cursor);
         uint32_t next_arr = __shfl_sync(kFull, ab.time, 0);
-        const uint32_t max_steps = p.max_steps;
-        const uint32_t all = own_mask<C>(x);
-        const bool ticks = EXT ? p.ticks != 0 : p.enable_mig != 0;
-        // Every pass of the loop below is one of three modes, which share one
-        // copy of each phase (iteration ends; finishes and copy stages;
-        // dispatch and tick; batch formation), so the hot loop stays small:
-        //   0: a window [tb, t1) in which every instance ends at most one
-        //      iteration: each lane ends and re-forms its own instances that
-        //      are in no migration ("solo"), each at its own time;
-        //   1: one step, at the next time tc < t1, of the window's instances
-        //      in a migration (both ends of every migration), in time order;
-        //   2: one step at the next global event (arrival, tick), or near the
-        //      step limit, over all instances.
-        bool in_cm = false;              // mode-1 steps of the current window remain
-        uint32_t t1 = 0, cm = 0;         // window end; own instances stepped in mode 1
-        uint32_t ucount = 0, u = kNone;  // distinct event times of the window; own solo time (C = 1)
-        uint32_t tlast = 0;              // latest event time processed in the window
-        for (;;) {
-            int mode;
-            uint32_t et[C];      // event time of each own instance in this pass
-            uint32_t heads = 0;  // own instances whose iteration ends in this pass
-            uint32_t tstep = 0;  // step time (modes 1 and 2)
-            bool tick = false;
-            if (in_cm) {
-                uint32_t cb = kNone;
+        if constexpr (kUnifiedLoop<C, SMS>) {
+            const uint32_t max_steps = p.max_steps;
+            const uint32_t all = own_mask<C>(x);
+            const bool ticks = EXT ? p.ticks != 0 : p.enable_mig != 0;
+            // Every pass of the loop below is one of three modes, which share one
+            // copy of each phase (iteration ends; finishes and copy stages;
+            // dispatch and tick; batch formation), so the hot loop stays small:
+            //   0: a window [tb, t1) in which every instance ends at most one
+            //      iteration: each lane ends and re-forms its own instances that
+            //      are in no migration ("solo"), each at its own time;
+            //   1: one step, at the next time tc < t1, of the window's instances
+            //      in a migration (both ends of every migration), in time order;
+            //   2: one step at the next global event (arrival, tick), or near the
+            //      step limit, over all instances.
+            bool in_cm = false;              // mode-1 steps of the current window remain
+            uint32_t t1 = 0, cm = 0;         // window end; own instances stepped in mode 1
+            uint32_t ucount = 0, u = kNone;  // distinct event times of the window; own solo time (C = 1)
+            uint32_t tlast = 0;              // latest event time processed in the window
+            for (;;) {
+                int mode;
+                uint32_t et[C];      // event time of each own instance in this pass
+                uint32_t heads = 0;  // own instances whose iteration ends in this pass
+                uint32_t tstep = 0;  // step time (modes 1 and 2)
+                bool tick = false;
+                if (in_cm) {
+                    uint32_t cb = kNone;
 #pragma unroll
-                for (int j = 0; j < C; ++j)
-                    if ((cm >> j) & 1u) cb = min(cb, x.busy[lane * C + j]);
-                const uint32_t tc = __reduce_min_sync(kFull, cb);
-                if (tc >= t1) {  // the window is complete
-                    in_cm = false;
-                    cn.steps += ucount;
-                    tmax = max(tmax, tlast);
-                    cn.finished = __shfl_sync(kFull, cn.finished, 0);  // finishes are all counted on lane 0
-                    cn.status = __reduce_min_sync(kFull, cn.status);
-                    if (cn.status < 0) break;
-                    continue;
+                    for (int j = 0; j < C; ++j)
+                        if ((cm >> j) & 1u) cb = min(cb, x.busy[lane * C + j]);
+                    const uint32_t tc = __reduce_min_sync(kFull, cb);
+                    if (tc >= t1) {  // the window is complete
+                        in_cm = false;
+                        cn.steps += ucount;
+                        tmax = max(tmax, tlast);
+                        cn.finished = __shfl_sync(kFull, cn.finished, 0);  // finishes are all counted on lane 0
+                        cn.status = __reduce_min_sync(kFull, cn.status);
+                        if (cn.status < 0) break;
+                        continue;
+                    }
+                    mode = 1;
+                    tstep = tc;
+                    tlast = max(tlast, tc);
+#pragma unroll
+                    for (int j = 0; j < C; ++j) {
+                        et[j] = tc;
+                        if (((cm >> j) & 1u) && x.busy[lane * C + j] == tc) heads |= 1u << j;
+                    }
+                } else {
+                    if (cn.finished == x.Q) { cn.status = SIM_REPLICA_DONE; break; }
+                    if (cn.steps == max_steps) break;
+                    uint32_t bz[C];
+                    uint32_t mb = kNone;
+#pragma unroll
+                    for (int j = 0; j < C; ++j) {
+                        const int i = lane * C + j;
+                        bz[j] = i < x.N ? x.busy[i] : kNone;
+                        mb = min(mb, bz[j]);
+                    }
+                    const uint32_t tb = __reduce_min_sync(kFull, mb);
+                    const uint32_t tg = ticks ? min(next_arr, next_tick) : next_arr;
+                    if (tb < tg && max_steps - cn.steps > (uint32_t)x.N) {
+                        mode = 0;
+                        t1 = (uint32_t)min((unsigned long long)tg, (unsigned long long)tb + (uint32_t)p.base);
+                        // instances with an iteration end in the window: stepped with
+                        // the others of a migration in time order (cm), or alone
+                        // (solo).  A destination whose source has no event in the
+                        // window is alone: only the source's events (stages, commit,
+                        // abort) touch the other end.
+                        cm = 0;
+                        uint32_t solo = 0;
+#pragma unroll
+                        for (int j = 0; j < C; ++j) {
+                            const int i = lane * C + j;
+                            et[j] = bz[j];
+                            if (bz[j] < t1) {
+                                const int role = x.mrole[i];
+                                if (role == MIG_NONE || (role == MIG_DST && x.busy[x.mpeer[i]] >= t1)) solo |= 1u << j;
+                                else cm |= 1u << j;
+                            }
+                        }
+                        heads = solo;
+                        tlast = 0;
+                        if (C == 1) {
+                            // distinct event times: one group per value of the solo times
+                            u = solo ? bz[0] : kNone;
+                            const uint32_t grp = __match_any_sync(kFull, u);
+                            ucount = __popc(__ballot_sync(kFull, u != kNone && (__ffs(grp) - 1) == lane));
+                            if (solo) tlast = bz[0];
+                        } else {
+                            for (uint32_t q = (uint32_t)lane; q < kHashSlots; q += 32) tset[q] = kNone;
+                            __syncwarp();
+                            uint32_t fresh = 0;
+#pragma unroll
+                            for (int j = 0; j < C; ++j) {
+                                if (!((solo >> j) & 1u)) continue;
+                                tlast = max(tlast, bz[j]);
+                                fresh += tset_insert(x, bz[j]);
+                            }
+                            ucount = __reduce_add_sync(kFull, fresh);
+                        }
+                    } else {
+                        mode = 2;
+                        const uint32_t tc = min(tb, next_arr);
+                        if (tc == kNone) { cn.status = SIM_ERR_DEADLOCK; break; }
+                        tick = ticks && next_tick <= tc;
+                        tstep = tick ? next_tick : tc;
+                        tmax = max(tmax, tstep);
+                        ++cn.steps;
+#pragma unroll
+                        for (int j = 0; j < C; ++j) {
+                            et[j] = tstep;
+                            if (bz[j] == tstep) heads |= 1u << j;
+                        }
+                    }
                 }
-                mode = 1;
-                tstep = tc;
-                tlast = max(tlast, tc);
+                // ---- 1. iteration ends: each lane ends its own instances' iterations ----
+                uint32_t fz = 0;  // own instances with a finishing request
 #pragma unroll
                 for (int j = 0; j < C; ++j) {
-                    et[j] = tc;
-                    if (((cm >> j) & 1u) && x.busy[lane * C + j] == tc) heads |= 1u << j;
+                    if (!((heads >> j) & 1u)) continue;
+                    x.t = et[j];
+                    if (inst_complete_head(x, lane * C + j)) fz |= 1u << j;
                 }
-            } else {
+                __syncwarp();
+                // ---- finishes and copy stages, instance by instance in ascending
+                // order, by the whole warp (in mode 0 only finishes, which touch
+                // their own instance alone, so their order does not matter) ----
+                const uint32_t visit = mode == 0 ? fz : heads;
+                for (uint32_t fl = __ballot_sync(kFull, visit != 0); fl; fl &= fl - 1) {
+                    const int l = __ffs(fl) - 1;
+                    const uint32_t vl = C == 1 ? 1u : __shfl_sync(kFull, visit, l);
+                    const uint32_t fzl = __shfl_sync(kFull, fz, l);
+                    for (uint32_t h = vl; h; h &= h - 1) {
+                        const int j = __ffs(h) - 1;
+                        const int i = l * C + j;
+                        x.t = __shfl_sync(kFull, pick_c<C>(et, j), l);
+                        if ((fzl >> j) & 1u) coop_finish(x, cn, i);
+                        if (mode != 0 && x.mrole[i] == MIG_SRC) coop_stage(x, cn, i);
+                    }
+                }
+                if (mode == 2) {
+                    x.t = tstep;
+                    if (next_arr == tstep) dispatch_phase<C, EXT>(x, cn, cursor, next_arr, ab);  // 2. dispatch
+                    if (tick) {  // 3. auto-scaling signal and migration tick
+                        const uint32_t nt = next_tick + p.interval;
+                        next_tick = nt < next_tick ? kNone : nt;  // saturate: no tick beyond 2^32 - 1
+                        if (EXT && p.autoscale) autoscale_tick<C>(x, cn, p);
+                        if (p.enable_mig) migration_tick<C, EXT>(x, cn, p.theta_num, p.theta_den);
+                    }
+                }
+                // ---- 4. batch formation: in mode 0 every lane forms its own solo
+                // instances at their own times; otherwise the idle instances with
+                // work are formed on lane 0 in ascending order (their preemptions
+                // may abort migrations, whose log records are lane 0's) ----
+                uint32_t want = 0;
+                if (mode == 0) {
+                    want = heads;
+                } else {
+                    const uint32_t mask = mode == 1 ? cm : all;
+#pragma unroll
+                    for (int j = 0; j < C; ++j) {
+                        const int i = lane * C + j;
+                        if (((mask >> j) & 1u) && x.busy[i] == kNone && (x.nrun[i] | x.wmask[i]) != 0) want |= 1u << j;
+                    }
+                }
+                for (uint32_t fl = mode == 0 ? 1u : __ballot_sync(kFull, want != 0); fl; fl &= fl - 1) {
+                    const int l = __ffs(fl) - 1;
+                    const uint32_t hl = mode == 0 ? want : (C == 1 ? 1u : __shfl_sync(kFull, want, l));
+                    const int owner = mode == 0 ? lane : l;
+                    if (mode == 0 || lane == 0) {
+                        for (uint32_t h = hl; h; h &= h - 1) {
+                            const int j = __ffs(h) - 1;
+                            x.t = mode == 0 ? pick_c<C>(et, j) : tstep;
+                            inst_form(x, cn, owner * C + j, p.base, p.a, p.b);
+                        }
+                    }
+                    __syncwarp();
+                }
+                // ---- step accounting ----
+                if (mode == 0) {
+                    if (__any_sync(kFull, cm != 0)) {
+                        // the window's instances in a migration next (both ends of
+                        // every migration, with or without an event of their own)
+#pragma unroll
+                        for (int j = 0; j < C; ++j) {
+                            const int i = lane * C + j;
+                            if (i < x.N && x.mrole[i] != MIG_NONE) cm |= 1u << j;
+                        }
+                        in_cm = true;
+                        continue;
+                    }
+                    cn.steps += ucount;
+                    tmax = max(tmax, tlast);
+                    cn.finished = __shfl_sync(kFull, cn.finished, 0);
+                    cn.status = __reduce_min_sync(kFull, cn.status);
+                    if (cn.status < 0) break;
+                } else if (mode == 1) {
+                    if (C == 1) {
+                        ucount += __any_sync(kFull, u == tstep) ? 0u : 1u;
+                    } else {
+                        uint32_t f2 = 0;
+                        if (lane == 0) f2 = tset_insert(x, tstep);
+                        ucount += __shfl_sync(kFull, f2, 0);
+                    }
+                    cn.status = __reduce_min_sync(kFull, cn.status);  // also a solo lane's error of this window
+                    if (cn.status < 0) {
+                        in_cm = false;
+                        cn.steps += ucount;
+                        tmax = max(tmax, tlast);
+                        cn.finished = __shfl_sync(kFull, cn.finished, 0);
+                        break;
+                    }
+                } else {
+                    cn.finished = __shfl_sync(kFull, cn.finished, 0);
+                    cn.status = __shfl_sync(kFull, cn.status, 0);
+                    if (cn.status < 0) break;
+                }
+            }
+            __syncwarp();
+        } else {
+            const uint32_t max_steps = p.max_steps;
+            const uint32_t all = own_mask<C>(x);
+            for (;;) {
                 if (cn.finished == x.Q) { cn.status = SIM_REPLICA_DONE; break; }
                 if (cn.steps == max_steps) break;
                 uint32_t bz[C];
@@ -1146,166 +1378,130 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, (!SMS && C <= 2) ? 8 : 4)
                     mb = min(mb, bz[j]);
                 }
                 const uint32_t tb = __reduce_min_sync(kFull, mb);
+                const bool ticks = EXT ? p.ticks != 0 : p.enable_mig != 0;
                 const uint32_t tg = ticks ? min(next_arr, next_tick) : next_arr;
                 if (tb < tg && max_steps - cn.steps > (uint32_t)x.N) {
-                    mode = 0;
-                    t1 = (uint32_t)min((unsigned long long)tg, (unsigned long long)tb + (uint32_t)p.base);
-                    // instances with an iteration end in the window: stepped with
-                    // the others of a migration in time order (cm), or alone
-                    // (solo).  A destination whose source has no event in the
-                    // window is alone: only the source's events (stages, commit,
-                    // abort) touch the other end.
-                    cm = 0;
-                    uint32_t solo = 0;
+                    // ---- window [tb, t1): at most one iteration end per instance ----
+                    const uint32_t t1 =
+                        (uint32_t)min((unsigned long long)tg, (unsigned long long)tb + (uint32_t)p.base);
+                    // instances with an iteration end in the window: stepped with the
+                    // others of a migration in time order (cm), or alone (solo).  A
+                    // destination whose source has no event in the window is alone:
+                    // only the source's events (stages, commit, abort) touch the other end.
+                    uint32_t cm = 0, solo = 0;
 #pragma unroll
                     for (int j = 0; j < C; ++j) {
                         const int i = lane * C + j;
-                        et[j] = bz[j];
                         if (bz[j] < t1) {
                             const int role = x.mrole[i];
                             if (role == MIG_NONE || (role == MIG_DST && x.busy[x.mpeer[i]] >= t1)) solo |= 1u << j;
                             else cm |= 1u << j;
                         }
                     }
-                    heads = solo;
-                    tlast = 0;
+                    if (C > 1) {
+                        for (uint32_t q = (uint32_t)lane; q < kHashSlots; q += 32) tset[q] = kNone;
+                        __syncwarp();
+                    }
+                    uint32_t fresh = 0;  // distinct event times this lane contributes (C > 1)
+                    uint32_t tlast = 0;  // latest event time processed in the window
+                    uint32_t fz = 0;     // this lane's instances with a finishing request
+#pragma unroll
+                    for (int j = 0; j < C; ++j) {
+                        if (!((solo >> j) & 1u)) continue;
+                        const int i = lane * C + j;
+                        x.t = bz[j];
+                        tlast = max(tlast, bz[j]);
+                        if (C > 1) fresh += tset_insert(x, bz[j]);
+                        if (inst_complete_head(x, i)) fz |= 1u << j;
+                    }
+                    // finishes, one instance at a time by the whole warp (they touch
+                    // only their own instance, so their order does not matter) ...
+                    for (uint32_t fl = __ballot_sync(kFull, fz != 0); fl; fl &= fl - 1) {
+                        const int l = __ffs(fl) - 1;
+                        for (uint32_t h = C == 1 ? 1u : __shfl_sync(kFull, fz, l); h; h &= h - 1) {
+                            const int j = __ffs(h) - 1;
+                            x.t = __shfl_sync(kFull, bz[j], l);
+                            coop_finish(x, cn, l * C + j);
+                        }
+                    }
+                    // ... then every lane forms its instances' next batches together
+#pragma unroll
+                    for (int j = 0; j < C; ++j) {
+                        if (!((solo >> j) & 1u)) continue;
+                        x.t = bz[j];
+                        inst_form(x, cn, lane * C + j, p.base, p.a, p.b);
+                    }
+                    __syncwarp();
+                    uint32_t ucount, u = kNone;
                     if (C == 1) {
-                        // distinct event times: one group per value of the solo times
                         u = solo ? bz[0] : kNone;
                         const uint32_t grp = __match_any_sync(kFull, u);
                         ucount = __popc(__ballot_sync(kFull, u != kNone && (__ffs(grp) - 1) == lane));
-                        if (solo) tlast = bz[0];
                     } else {
-                        for (uint32_t q = (uint32_t)lane; q < kHashSlots; q += 32) tset[q] = kNone;
-                        __syncwarp();
-                        uint32_t fresh = 0;
-#pragma unroll
-                        for (int j = 0; j < C; ++j) {
-                            if (!((solo >> j) & 1u)) continue;
-                            tlast = max(tlast, bz[j]);
-                            fresh += tset_insert(x, bz[j]);
-                        }
                         ucount = __reduce_add_sync(kFull, fresh);
                     }
-                } else {
-                    mode = 2;
-                    const uint32_t tc = min(tb, next_arr);
-                    if (tc == kNone) { cn.status = SIM_ERR_DEADLOCK; break; }
-                    tick = ticks && next_tick <= tc;
-                    tstep = tick ? next_tick : tc;
-                    tmax = max(tmax, tstep);
-                    ++cn.steps;
+                    // instances in a migration (both ends, with or without an event
+                    // of their own in the window): steps in time order on lane 0
+                    if (__any_sync(kFull, cm != 0)) {
 #pragma unroll
-                    for (int j = 0; j < C; ++j) {
-                        et[j] = tstep;
-                        if (bz[j] == tstep) heads |= 1u << j;
+                        for (int j = 0; j < C; ++j) {
+                            const int i = lane * C + j;
+                            if (i < x.N && x.mrole[i] != MIG_NONE) cm |= 1u << j;
+                        }
+                        for (;;) {
+                            uint32_t cb = kNone;
+#pragma unroll
+                            for (int j = 0; j < C; ++j)
+                                if ((cm >> j) & 1u) cb = min(cb, x.busy[lane * C + j]);
+                            const uint32_t tc = __reduce_min_sync(kFull, cb);
+                            if (tc >= t1) break;
+                            x.t = tc;
+                            tlast = max(tlast, tc);
+                            complete_all<C>(x, cn, cm);
+                            form_all<C>(x, cn, cm, p);
+                            if (C == 1) {
+                                ucount += __any_sync(kFull, u == tc) ? 0u : 1u;
+                            } else {
+                                uint32_t f2 = 0;
+                                if (lane == 0) f2 = tset_insert(x, tc);
+                                ucount += __shfl_sync(kFull, f2, 0);
+                            }
+                            cn.status = __shfl_sync(kFull, cn.status, 0);
+                            if (cn.status < 0) break;
+                        }
                     }
+                    cn.steps += ucount;
+                    tmax = max(tmax, tlast);  // x.t is set again before any further use
+                    cn.finished = __shfl_sync(kFull, cn.finished, 0);  // finishes are all counted on lane 0
+                    const int ws = __reduce_min_sync(kFull, cn.status);
+                    cn.status = ws;
+                    if (cn.status < 0) break;
+                    continue;
                 }
-            }
-            // ---- 1. iteration ends: each lane ends its own instances' iterations ----
-            uint32_t fz = 0;  // own instances with a finishing request
-#pragma unroll
-            for (int j = 0; j < C; ++j) {
-                if (!((heads >> j) & 1u)) continue;
-                x.t = et[j];
-                if (inst_complete_head(x, lane * C + j)) fz |= 1u << j;
-            }
-            __syncwarp();
-            // ---- finishes and copy stages, instance by instance in ascending
-            // order, by the whole warp (in mode 0 only finishes, which touch
-            // their own instance alone, so their order does not matter) ----
-            const uint32_t visit = mode == 0 ? fz : heads;
-            for (uint32_t fl = __ballot_sync(kFull, visit != 0); fl; fl &= fl - 1) {
-                const int l = __ffs(fl) - 1;
-                const uint32_t vl = C == 1 ? 1u : __shfl_sync(kFull, visit, l);
-                const uint32_t fzl = __shfl_sync(kFull, fz, l);
-                for (uint32_t h = vl; h; h &= h - 1) {
-                    const int j = __ffs(h) - 1;
-                    const int i = l * C + j;
-                    x.t = __shfl_sync(kFull, pick_c<C>(et, j), l);
-                    if ((fzl >> j) & 1u) coop_finish(x, cn, i);
-                    if (mode != 0 && x.mrole[i] == MIG_SRC) coop_stage(x, cn, i);
-                }
-            }
-            if (mode == 2) {
-                x.t = tstep;
-                if (next_arr == tstep) dispatch_phase<C, EXT>(x, cn, cursor, next_arr, ab);  // 2. dispatch
+                // ---- one step at the next event time (global events, or near the step limit) ----
+                const uint32_t tc = min(tb, next_arr);
+                if (tc == kNone) { cn.status = SIM_ERR_DEADLOCK; break; }
+                const bool tick = ticks && next_tick <= tc;
+                x.t = tick ? next_tick : tc;
+                tmax = max(tmax, x.t);
+                ++cn.steps;
+                const uint32_t f1 = cn.finished;
+                if (tb == x.t) complete_all<C>(x, cn, all);  // 1. iteration ends
+                cn.finished = __shfl_sync(kFull, cn.finished, 0);
+                if (next_arr == x.t) dispatch_phase<C, EXT>(x, cn, cursor, next_arr, ab);  // 2. dispatch
                 if (tick) {  // 3. auto-scaling signal and migration tick
                     const uint32_t nt = next_tick + p.interval;
                     next_tick = nt < next_tick ? kNone : nt;  // saturate: no tick beyond 2^32 - 1
                     if (EXT && p.autoscale) autoscale_tick<C>(x, cn, p);
                     if (p.enable_mig) migration_tick<C, EXT>(x, cn, p.theta_num, p.theta_den);
                 }
-            }
-            // ---- 4. batch formation: in mode 0 every lane forms its own solo
-            // instances at their own times; otherwise the idle instances with
-            // work are formed on lane 0 in ascending order (their preemptions
-            // may abort migrations, whose log records are lane 0's) ----
-            uint32_t want = 0;
-            if (mode == 0) {
-                want = heads;
-            } else {
-                const uint32_t mask = mode == 1 ? cm : all;
-#pragma unroll
-                for (int j = 0; j < C; ++j) {
-                    const int i = lane * C + j;
-                    if (((mask >> j) & 1u) && x.busy[i] == kNone && (x.nrun[i] | x.wmask[i]) != 0) want |= 1u << j;
-                }
-            }
-            for (uint32_t fl = mode == 0 ? 1u : __ballot_sync(kFull, want != 0); fl; fl &= fl - 1) {
-                const int l = __ffs(fl) - 1;
-                const uint32_t hl = mode == 0 ? want : (C == 1 ? 1u : __shfl_sync(kFull, want, l));
-                const int owner = mode == 0 ? lane : l;
-                if (mode == 0 || lane == 0) {
-                    for (uint32_t h = hl; h; h &= h - 1) {
-                        const int j = __ffs(h) - 1;
-                        x.t = mode == 0 ? pick_c<C>(et, j) : tstep;
-                        inst_form(x, cn, owner * C + j, p.base, p.a, p.b);
-                    }
-                }
-                __syncwarp();
-            }
-            // ---- step accounting ----
-            if (mode == 0) {
-                if (__any_sync(kFull, cm != 0)) {
-                    // the window's instances in a migration next (both ends of
-                    // every migration, with or without an event of their own)
-#pragma unroll
-                    for (int j = 0; j < C; ++j) {
-                        const int i = lane * C + j;
-                        if (i < x.N && x.mrole[i] != MIG_NONE) cm |= 1u << j;
-                    }
-                    in_cm = true;
-                    continue;
-                }
-                cn.steps += ucount;
-                tmax = max(tmax, tlast);
-                cn.finished = __shfl_sync(kFull, cn.finished, 0);
-                cn.status = __reduce_min_sync(kFull, cn.status);
-                if (cn.status < 0) break;
-            } else if (mode == 1) {
-                if (C == 1) {
-                    ucount += __any_sync(kFull, u == tstep) ? 0u : 1u;
-                } else {
-                    uint32_t f2 = 0;
-                    if (lane == 0) f2 = tset_insert(x, tstep);
-                    ucount += __shfl_sync(kFull, f2, 0);
-                }
-                cn.status = __reduce_min_sync(kFull, cn.status);  // also a solo lane's error of this window
-                if (cn.status < 0) {
-                    in_cm = false;
-                    cn.steps += ucount;
-                    tmax = max(tmax, tlast);
-                    cn.finished = __shfl_sync(kFull, cn.finished, 0);
-                    break;
-                }
-            } else {
-                cn.finished = __shfl_sync(kFull, cn.finished, 0);
+                form_all<C>(x, cn, all, p);  // 4. batch formation
+                (void)f1;
                 cn.status = __shfl_sync(kFull, cn.status, 0);
                 if (cn.status < 0) break;
             }
+            __syncwarp();
         }
-        __syncwarp();
         // fold the other lanes' counters into lane 0's
         const uint32_t tfin = __reduce_max_sync(kFull, tmax);
         const uint32_t a_pre = __reduce_add_sync(kFull, l0 ? 0u : cn.preemptions);
