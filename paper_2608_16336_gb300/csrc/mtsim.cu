@@ -428,8 +428,8 @@ __device__ __forceinline__ void coop_finish(const Ctx &x, Cnt &cn, int i) {
     const int p0 = __popc(e0 & below), p1 = __popc(e0) + __popc(e1 & below);
     const uint32_t fm = __reduce_min_sync(kFull, min(k0 ? sl_fin(a0) : kNone, k1 ? sl_fin(a1) : kNone));
     __syncwarp();
-    if (k0) p[p0] = a0;
-    if (k1) p[p1] = a1;
+    if (k0 && p0 != q0) p[p0] = a0;  // only the records that move are written
+    if (k1 && p1 != q1) p[p1] = a1;
     if (x.lane == 0) {
         const uint32_t nfin = __popc(m0) + __popc(m1);
         x.free_[i] += freed;
