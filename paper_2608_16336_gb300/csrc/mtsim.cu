@@ -235,9 +235,9 @@ __device__ __forceinline__ int arg_ext(const Ctx &x, uint32_t el, bool want_max,
         }
     }
     const int m = want_max ? __reduce_max_sync(kFull, bv) : __reduce_min_sync(kFull, bv);
-    const uint32_t eq = __ballot_sync(kFull, bi >= 0 && bv == m);
-    if (!eq) return -1;
-    return __shfl_sync(kFull, bi, __ffs(eq) - 1);
+    // lowest instance among those at the extreme (INT_MAX: none)
+    const int best = __reduce_min_sync(kFull, (bi >= 0 && bv == m) ? bi : INT_MAX);
+    return best == INT_MAX ? -1 : best;
 }
 
 // ---- single-thread instance logic (no collectives inside) -------------------
@@ -747,8 +747,7 @@ __device__ __forceinline__ void dispatch_phase(const Ctx &x, Cnt &cn, uint32_t &
             }
         }
         const int m = __reduce_max_sync(kFull, bv);
-        const uint32_t em = __ballot_sync(kFull, bi >= 0 && bv == m);
-        const int best = __shfl_sync(kFull, bi, __ffs(em) - 1);
+        const int best = __reduce_min_sync(kFull, (bi >= 0 && bv == m) ? bi : INT_MAX);
         dispatch_to(x, cn, best, ab.pb + (uint32_t)l, (int)k1, po & 0xFFFFu, po >> 16, false);
         __syncwarp();
         cursor += 1u;
