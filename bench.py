@@ -191,13 +191,16 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
-def sized_simulator(mtsim, w, cap: int, stream):
+def sized_simulator(mtsim, w, cap: int, stream, order=None):
     """A simulator whose migration log holds every record of every replica:
     one complete run with capacity ``cap``; if some replica produced more
-    records, the simulator is rebuilt with exactly enough room.  Returns the
+    records, the simulator is rebuilt with exactly enough room.  ``order``:
+    the replicas' start order (sim_set_order), or None.  Returns the
     simulator (after that run), its capacity and the run's stats."""
     while True:
         sim = mtsim.Simulator(w, event_log_capacity=cap, stream=stream)
+        if order is not None:
+            sim.set_order(order)
         sim.load(on_device=True)
         mtsim.sim_run(sim.handle, 1 << 62, False)
         st = sim.stats()
@@ -261,10 +264,13 @@ def bench_gpu(args):
 
     cid = args.workload
     r_all = args.replicas or workloads.num_replicas(cid)
-    lo, hi = workloads.partition(workloads.predicted_work(cid, args.requests)[:r_all], ws)[rank]
+    work = workloads.predicted_work(cid, args.requests)[:r_all]
+    lo, hi = workloads.partition(work, ws)[rank]
     w = workloads.config(cid, replicas=range(lo, hi), requests=args.requests)
     stream = torch.cuda.current_stream()
-    sim, cap, st0 = sized_simulator(mtsim, w, args.log_capacity or initial_log_capacity(w), stream)
+    # replicas with the most predicted work start first (ties: trace order)
+    order = None if args.trace_order else np.argsort(-work[lo:hi], kind="stable").astype(np.int32)
+    sim, cap, st0 = sized_simulator(mtsim, w, args.log_capacity or initial_log_capacity(w), stream, order)
     R, Q = w.num_replicas, w.total_requests
 
     clocks = ClockSampler(local, args.clocks_dir)
@@ -356,6 +362,7 @@ def bench_gpu(args):
             "migration_log_records": int(st["log_events"].sum()),
             "max_log_records_per_replica": int(st["log_events"].max()),
             "parallelism": "replicas partitioned across GPUs by predicted work, no collective on the data path",
+            "replica_order": "trace order" if args.trace_order else "descending predicted work (requests x instances x load), ties in trace order",
             "l2": "inputs larger than L2: trace %.0f MB + per-request state %.0f MB resident" % (
                 Q * 9 / 1e6, Q * 32 / 1e6),
         },
@@ -394,9 +401,11 @@ def bench_gpu(args):
 
 def bench_other(torch, mtsim, workloads, cid: int, stream, args) -> dict:
     """One smaller workload at full size, timed the same way (3 warm-up and
-    3 timed complete simulations, every log record kept)."""
+    3 timed complete simulations, every log record kept, the same replica
+    order rule)."""
     w = workloads.config(cid)
-    sim, cap, _ = sized_simulator(mtsim, w, initial_log_capacity(w), stream)
+    order = None if args.trace_order else np.argsort(-workloads.predicted_work(cid), kind="stable").astype(np.int32)
+    sim, cap, _ = sized_simulator(mtsim, w, initial_log_capacity(w), stream, order)
     dev_s, k_s, _ = time_device_steps(torch, mtsim, sim, stream, 3, 3)
     st = sim.stats()
     launch = sim.launch_info()
@@ -515,6 +524,8 @@ def main():
     ap.add_argument("--cpu-replicas-per-step", type=int, default=64)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-others", action="store_true", help="skip the smaller workloads' lines")
+    ap.add_argument("--trace-order", action="store_true",
+                    help="start replicas in trace order instead of by descending predicted work")
     ap.add_argument("--clocks-dir", default=os.path.join(tempfile.gettempdir(), "mtsim_bench"),
                     help="where the raw nvidia-smi clock samples of the timed region are written")
     ap.add_argument("--replicas", type=int, default=0, help="profiling only: first N replicas of the workload")

@@ -252,6 +252,17 @@ int sim_reset(sim_t *sim);
  * allocated.  sim_run_static has no drain schedule. */
 int sim_set_drain(sim_t *sim, const uint32_t *drain_start_us, int on_device);
 
+/* Sets the order in which sim_run starts replicas: the persistent grid takes
+ * replicas from a counter, and with an order set the k-th replica taken is
+ * order[k].  Starting the replicas with the most work first shortens the
+ * tail of a launch that runs more replicas than fit on the GPU at once.
+ * Results never depend on the order.  order: host, [R], a permutation of
+ * 0..R-1 (checked: anything else returns SIM_ERR_ARG and keeps the previous
+ * order); copied, so the buffer may be reused when the call returns.  NULL
+ * restores trace order.  Takes effect at the next sim_run.  The paper has no
+ * counterpart; this is a scheduling aid of the batched simulation. */
+int sim_set_order(sim_t *sim, const int32_t *order);
+
 /* Advances every unfinished replica by at most max_steps_per_replica steps
  * (>= 1) in one persistent kernel launch; a later call resumes where this one
  * stopped.  If num_unfinished (host) is non-NULL the call synchronises and

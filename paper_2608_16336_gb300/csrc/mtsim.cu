@@ -141,6 +141,7 @@ struct Params {
     RepState *rep;
     sim_migration_event_t *log;
     int *work;
+    const int *order;             // [R] start order of the replicas, or NULL (trace order)
 };
 
 // Per-warp view of the replica being simulated: instance state in shared
@@ -1082,7 +1083,10 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, (!SMS && C <= 2) ? 8 : 4)
     uint32_t *tset = reinterpret_cast<uint32_t *>(blob + p.L.bytes + slot_bytes);
     for (;;) {
         int r = 0;
-        if (lane == 0) r = atomicAdd(p.work, 1);
+        if (lane == 0) {
+            r = atomicAdd(p.work, 1);
+            if (p.order && r < p.R) r = p.order[r];
+        }
         r = __shfl_sync(kFull, r, 0);
         if (r >= p.R) break;
         const RepState rs = p.rep[r];
@@ -1796,6 +1800,7 @@ struct sim {
     uint4 *d_node = nullptr;
     sim_request_result_t *d_res = nullptr;
     uint32_t *d_drain = nullptr;  // [R][N] drain start times (sim_set_drain), or NULL
+    int *d_order = nullptr;       // [R] replica start order (sim_set_order), or NULL
     uint32_t *d_ftc = nullptr;    // [R] first-token counts for sim_metrics
     sim_latency_stats_t *d_lat = nullptr;  // device staging of sim_latency_stats for host output
     int *d_lat_rep = nullptr;              // chunk table of sim_latency_stats: replica and first record
@@ -1911,6 +1916,7 @@ mt::Params make_params(const sim_t *s, long long max_steps) {
     p.rep = s->d_rep;
     p.log = s->d_log;
     p.work = s->d_work;
+    p.order = s->d_order;
     return p;
 }
 
@@ -2242,6 +2248,31 @@ int sim_set_drain(sim_t *s, const uint32_t *drain_start_us, int on_device) {
                                     on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice, s->stream);
     if (e == cudaSuccess && !on_device) e = cudaStreamSynchronize(s->stream);  // the host buffer may be reused
     if (e != cudaSuccess) return cuda_fail(s, e, "sim_set_drain copy");
+    return SIM_OK;
+}
+
+int sim_set_order(sim_t *s, const int32_t *order) {
+    if (!s) return SIM_ERR_ARG;
+    if (!order) {
+        dfree(s, s->d_order);
+        s->d_order = nullptr;
+        return SIM_OK;
+    }
+    const int R = s->cl.num_replicas;
+    std::vector<char> seen((size_t)R, 0);
+    for (int k = 0; k < R; ++k) {
+        const int32_t r = order[k];
+        if (r < 0 || r >= R || seen[(size_t)r])
+            return fail(s, SIM_ERR_ARG, "order is not a permutation of 0..%d (entry %d = %d)", R - 1, k, (int)r);
+        seen[(size_t)r] = 1;
+    }
+    if (!s->d_order) {
+        s->d_order = (int *)dalloc(s, (size_t)R * 4);
+        if (!s->d_order) return fail(s, SIM_ERR_OOM, "device allocation of the replica order failed");
+    }
+    cudaError_t e = cudaMemcpyAsync(s->d_order, order, (size_t)R * 4, cudaMemcpyHostToDevice, s->stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s->stream);  // the host buffer may be reused
+    if (e != cudaSuccess) return cuda_fail(s, e, "sim_set_order copy");
     return SIM_OK;
 }
 

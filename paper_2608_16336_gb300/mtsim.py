@@ -81,7 +81,7 @@ class sim_allocator_t(ctypes.Structure):
 
 EXPORTS = ["sim_create", "sim_load_trace", "sim_reset", "sim_run", "sim_metrics", "sim_destroy",
            "sim_last_error", "sim_strerror", "sim_device_bytes", "sim_run_static", "sim_set_drain",
-           "sim_latency_stats", "sim_launch_info"]
+           "sim_latency_stats", "sim_launch_info", "sim_set_order"]
 SIM_STATIC_SCRATCH_BYTES = 32 << 20
 
 _LIB = None
@@ -121,6 +121,8 @@ def lib() -> ctypes.CDLL:
         L.sim_strerror.restype = ctypes.c_char_p
         L.sim_device_bytes.argtypes = [vp]
         L.sim_device_bytes.restype = ctypes.c_size_t
+        L.sim_set_order.argtypes = [vp, vp]
+        L.sim_set_order.restype = ctypes.c_int
         L.sim_launch_info.argtypes = [vp, ctypes.POINTER(sim_launch_info_t)]
         L.sim_launch_info.restype = ctypes.c_int
         L.sim_run_static.argtypes = [ctypes.POINTER(sim_cluster_t), ctypes.POINTER(sim_tier_table_t),
@@ -195,6 +197,10 @@ def sim_destroy(handle) -> None:
 
 def sim_device_bytes(handle) -> int:
     return int(lib().sim_device_bytes(handle))
+
+
+def sim_set_order(handle, order_ptr) -> int:
+    return _check(lib().sim_set_order(handle, order_ptr), handle)
 
 
 def sim_launch_info(handle) -> dict:
@@ -322,6 +328,16 @@ class Simulator:
         st = np.empty(self.w.num_replicas, STATS_DTYPE)
         sim_metrics(self.handle, None, st.ctypes.data, None, 0)
         return st
+
+    def set_order(self, order) -> None:
+        """Replica start order (a permutation of 0..R-1), or None for trace order."""
+        if order is None:
+            sim_set_order(self.handle, None)
+            return
+        self._order = np.ascontiguousarray(order, np.int32)
+        if self._order.shape != (self.w.num_replicas,):
+            raise ValueError("order must have one entry per replica")
+        sim_set_order(self.handle, self._order.ctypes.data)
 
     def launch_info(self) -> dict:
         return sim_launch_info(self.handle)

@@ -211,6 +211,33 @@ def test_migration_threshold_equality():
         assert (st["migration_starts"] > 0).all() == (num == 0)
 
 
+def test_replica_start_order_changes_nothing():
+    """Starting the replicas in another order (sim_set_order) gives the same
+    results bit for bit, with more replicas than the GPU holds at once (so
+    the reordered counter feeds several waves); a non-permutation is
+    rejected and leaves the previous order."""
+    w = W.config(4, replicas=range(3000), requests=300)
+    want = parity.run_gpu(w, event_log_capacity=1024)
+    perm = np.random.default_rng(7).permutation(w.num_replicas)
+    sim = mtsim.Simulator(w, event_log_capacity=1024)
+    try:
+        with pytest.raises(mtsim.SimError) as e:
+            sim.set_order(np.zeros(w.num_replicas, np.int32))
+        assert e.value.code == mtsim.SIM_ERR_ARG
+        sim.set_order(perm)
+        sim.load()
+        assert sim.launch_info()["grid_blocks"] * 2 < w.num_replicas
+        assert sim.run() == 0
+        res, st, ev = sim.metrics()
+        events = [sim.events_of(ev, st, r) for r in range(w.num_replicas)]
+        sim.set_order(None)
+    finally:
+        sim.close()
+    assert (res == want[0]).all() and (st == want[1]).all()
+    for a, b in zip(events, want[2]):
+        np.testing.assert_array_equal(a, b)
+
+
 # ----------------------------------------------------------- full size --
 def test_workload1_full_size_sampled():
     """The 1,024-replica workload at full size, in the launch configuration
@@ -259,7 +286,9 @@ def test_workload4_full_size_sampled():
     import torch
 
     w = W.config(4)
-    sim, cap, st0 = bench.sized_simulator(mtsim, w, bench.initial_log_capacity(w), torch.cuda.current_stream())
+    order = np.argsort(-W.predicted_work(4), kind="stable").astype(np.int32)  # the benchmark's start order
+    sim, cap, st0 = bench.sized_simulator(mtsim, w, bench.initial_log_capacity(w), torch.cuda.current_stream(),
+                                          order)
     try:
         assert sim.launch_info()["instances_per_lane"] == 2 and not sim.launch_info()["slots_in_shared"]
         res, st, ev = sim.metrics()
