@@ -52,6 +52,10 @@ class OracleConfig(ctypes.Structure):
         ("scale_den", ctypes.c_int32),
         ("pad_", ctypes.c_int32),
         ("drain_start_us", ctypes.c_void_p),
+        ("n_headroom_changes", ctypes.c_int32),
+        ("pad2_", ctypes.c_int32),
+        ("headroom_change_step", ctypes.c_void_p),
+        ("headroom_change_table", ctypes.c_void_p),
     ]
 
 
@@ -137,9 +141,12 @@ def make_config(num_instances, blocks_per_instance, headroom, *, tokens_per_bloc
                 iter_base_us=4000, iter_us_per_prefill_token=20, iter_us_per_decode_seq=30,
                 migrate_blocks_per_iter=64, enable_migration=1, migrate_interval_us=50_000,
                 theta_num=3, theta_den=10, check_invariants=0, autoscale=0, scale_out_num=-1, scale_in_num=3,
-                scale_den=2, drain_start_us=None) -> OracleConfig:
+                scale_den=2, drain_start_us=None, headroom_schedule=None) -> OracleConfig:
     """A replica's configuration; ``drain_start_us`` ([num_instances] times,
-    NONE32 = never) is kept alive on the returned object as ``_drain``."""
+    NONE32 = never) is kept alive on the returned object as ``_drain``.
+    ``headroom_schedule``: [(step, table)] — before the step of that index
+    (0-based) is processed, the headroom table becomes ``table``; its arrays
+    are kept alive as ``_sched``."""
     c = OracleConfig()
     c.num_instances = num_instances
     c.blocks_per_instance = blocks_per_instance
@@ -167,10 +174,22 @@ def make_config(num_instances, blocks_per_instance, headroom, *, tokens_per_bloc
         if c._drain.shape != (num_instances,):
             raise ValueError("drain_start_us needs one time per instance")
         c.drain_start_us = c._drain.ctypes.data
+    c._sched = None
+    if headroom_schedule:
+        steps = np.ascontiguousarray([int(st) for st, _ in headroom_schedule], np.int64)
+        tables = np.zeros((len(headroom_schedule), MAXK), np.int32)
+        for j, (_, tab) in enumerate(headroom_schedule):
+            if len(tab) != len(headroom):
+                raise ValueError("every scheduled table needs one entry per tier")
+            tables[j, : len(tab)] = tab
+        c._sched = (steps, tables)
+        c.n_headroom_changes = len(headroom_schedule)
+        c.headroom_change_step = steps.ctypes.data
+        c.headroom_change_table = tables.ctypes.data
     return c
 
 
-def config_for(w, r: int, check_invariants: int = 0) -> OracleConfig:
+def config_for(w, r: int, check_invariants: int = 0, headroom_schedule=None) -> OracleConfig:
     return make_config(
         w.num_instances, w.blocks_per_instance, w.tables_h[int(w.replica_table[r])],
         tokens_per_block=w.tokens_per_block, max_batch=w.max_batch, iter_base_us=w.iter_base_us,
@@ -180,7 +199,8 @@ def config_for(w, r: int, check_invariants: int = 0) -> OracleConfig:
         check_invariants=check_invariants, autoscale=getattr(w, "autoscale", 0),
         scale_out_num=getattr(w, "scale_out_num", -1), scale_in_num=getattr(w, "scale_in_num", 3),
         scale_den=getattr(w, "scale_den", 2),
-        drain_start_us=None if getattr(w, "drain_start_us", None) is None else w.drain_start_us[r])
+        drain_start_us=None if getattr(w, "drain_start_us", None) is None else w.drain_start_us[r],
+        headroom_schedule=headroom_schedule)
 
 
 class ReplicaResult:
@@ -236,8 +256,10 @@ def run_trace(cfg: OracleConfig, arrival, plen, olen, tier, *, max_steps: int = 
 
 
 def run_workload(w, replicas=None, *, nthreads: int = 1, max_steps: int = 1 << 62, log_capacity: int = 1 << 16,
-                 check_invariants: int = 0, so_path: str | None = None) -> dict[int, ReplicaResult]:
-    """Simulates the chosen replicas of workload ``w``; returns {replica: result}."""
+                 check_invariants: int = 0, so_path: str | None = None,
+                 headroom_schedules: dict | None = None) -> dict[int, ReplicaResult]:
+    """Simulates the chosen replicas of workload ``w``; returns {replica: result}.
+    ``headroom_schedules``: {replica: [(step, table)]} (see make_config)."""
     reps = list(range(w.num_replicas)) if replicas is None else [int(r) for r in replicas]
     n = len(reps)
     cfgs = (OracleConfig * max(n, 1))()
@@ -249,8 +271,9 @@ def run_workload(w, replicas=None, *, nthreads: int = 1, max_steps: int = 1 << 6
         res = ReplicaResult(sl.stop - sl.start, log_capacity)
         io, k = _io_for(w.arrival_us[sl], w.prompt_len[sl], w.output_len[sl], w.tier[sl], res)
         keep.append(k)
-        cfg = config_for(w, r, check_invariants)
+        cfg = config_for(w, r, check_invariants, (headroom_schedules or {}).get(r))
         keep.append(cfg._drain)
+        keep.append(cfg._sched)
         cfgs[j] = cfg
         ios[j] = io
         results[r] = res

@@ -90,6 +90,15 @@ typedef struct {
     int32_t scale_out_num, scale_in_num, scale_den;  /* thresholds on the mean F_normal */
     int32_t pad_;
     const uint32_t *drain_start_us;  /* [num_instances] or NULL: instance i drains from that time on */
+    /* Headroom schedule (adaptive headroom, Sec. 6 "Adaptive headroom
+     * allocation"): change j replaces the table H by
+     * headroom_change_table[j * MAXK .. + num_tiers) just before the step of
+     * index headroom_change_step[j] (0-based count of the steps processed so
+     * far) is processed.  Steps non-decreasing; 0 changes = the static table. */
+    int32_t n_headroom_changes;
+    int32_t pad2_;
+    const int64_t *headroom_change_step;   /* [n_headroom_changes] */
+    const int32_t *headroom_change_table;  /* [n_headroom_changes * MAXK] */
 } oracle_config_t;
 
 typedef struct {
@@ -166,6 +175,8 @@ struct Sim {
     int64_t cursor = 0;           /* next request not yet arrived */
     int64_t next_tick = 0;
     uint32_t now = 0;
+    int32_t H[MAXK];              /* the headroom table in force (c.headroom, then the schedule's) */
+    int32_t next_change = 0;      /* next entry of the headroom schedule */
 
     Sim(const oracle_config_t &cfg, oracle_io_t &o, oracle_stats_t &s) : c(cfg), io(o), st(s) {}
 
@@ -185,7 +196,7 @@ struct Sim {
         int h = hol_request(in);
         if (h >= 0) usage += need_blocks(req[h]);                      /* HoL demand; other queued: 0 */
         for (int k = 0; k < c.num_tiers; ++k)
-            if (in.cnt[k] > 0) usage += c.headroom[k];                 /* H_k once per present tier */
+            if (in.cnt[k] > 0) usage += H[k];                          /* H_k once per present tier */
         usage += in.reserved_in;                                       /* inbound migration copy */
         num = (int64_t)c.blocks_per_instance - usage;
         den = in.running.empty() ? 1 : (int64_t)in.running.size();
@@ -581,6 +592,14 @@ struct Sim {
             return false;
         for (int k = 0; k < c.num_tiers; ++k)
             if (c.headroom[k] < 0) return false;
+        if (c.n_headroom_changes < 0 || (c.n_headroom_changes > 0 && (!c.headroom_change_step || !c.headroom_change_table)))
+            return false;
+        for (int j = 0; j < c.n_headroom_changes; ++j) {
+            if (c.headroom_change_step[j] < 0 || (j > 0 && c.headroom_change_step[j] < c.headroom_change_step[j - 1]))
+                return false;
+            for (int k = 0; k < c.num_tiers; ++k)
+                if (c.headroom_change_table[j * MAXK + k] < 0) return false;
+        }
         return true;
     }
     bool validate_trace() const {
@@ -618,9 +637,15 @@ struct Sim {
             in.cnt.assign(c.num_tiers, 0);
         }
         next_tick = c.migrate_interval_us;
+        for (int k = 0; k < MAXK; ++k) H[k] = k < c.num_tiers ? c.headroom[k] : 0;
         st.status = ST_INCOMPLETE;
         while (st.finished < io.nreq) {
             if (st.steps >= max_steps) return;
+            /* headroom changes due before this step (adaptive headroom) */
+            while (next_change < c.n_headroom_changes && c.headroom_change_step[next_change] <= st.steps) {
+                for (int k = 0; k < c.num_tiers; ++k) H[k] = c.headroom_change_table[next_change * MAXK + k];
+                ++next_change;
+            }
             const int64_t INF = INT64_MAX;
             int64_t t = cursor < io.nreq ? (int64_t)io.arrival_us[cursor] : INF;
             for (const Inst &in : inst)

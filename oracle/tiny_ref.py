@@ -36,10 +36,13 @@ def _ceil_div(a: int, b: int) -> int:
 class TinySim:
     def __init__(self, n, m, headroom, trace, *, t_blk=16, bmax=64, base=4000, a=20, b=30, s_blocks=64,
                  migration=True, interval=50_000, theta=Fraction(3, 10), binary=False, binary_h=0,
-                 drain=None, autoscale=False, scale_out=Fraction(-1, 2), scale_in=Fraction(3, 2)):
+                 drain=None, autoscale=False, scale_out=Fraction(-1, 2), scale_in=Fraction(3, 2),
+                 headroom_schedule=None):
         self.N, self.M, self.T, self.Bmax = n, m, t_blk, bmax
         self.H = list(headroom)
         self.K = len(self.H)
+        # adaptive headroom: [(step, table)], table in force from the step of that index on
+        self.schedule = sorted(headroom_schedule or [], key=lambda e: e[0])
         self.base, self.a, self.b, self.S = base, a, b, s_blocks
         self.migration, self.interval, self.theta = migration, interval, theta
         self.binary, self.binary_h = binary, binary_h
@@ -269,6 +272,9 @@ class TinySim:
         nxt = 0
         tick = self.interval
         while sum(1 for x in self.out["finish"] if x != NONE32) < q and self.steps < max_steps:
+            for step, table in self.schedule:
+                if step == self.steps:
+                    self.H = list(table)
             cands = [bu for bu in self.busy_until if bu is not None]
             if nxt < q:
                 cands.append(self.trace[nxt][0])

@@ -6,6 +6,7 @@ import numpy as np
 import pytest
 
 from oracle import oracle as O
+from tests import test_oracle_adaptive as adpins
 from tests import test_oracle_autoscale as apins
 from tests import test_oracle_pins as pins
 
@@ -13,7 +14,7 @@ MUTANTS = {
     "drop HoL demand (Eq. 2)": ("if (h >= 0) usage += need_blocks(req[h]);                      /* HoL demand",
                                 "(void)h;  /* HoL demand"),
     "headroom per request instead of per tier (Eq. 4)": (
-        "if (in.cnt[k] > 0) usage += c.headroom[k];", "usage += (int64_t)c.headroom[k] * in.cnt[k];"),
+        "if (in.cnt[k] > 0) usage += H[k];", "usage += (int64_t)H[k] * in.cnt[k];"),
     "drop inbound reservation": ("usage += in.reserved_in;                                       /* inbound",
                                  "/* inbound"),
     "dispatch ties to highest index": ("if (!draining(i) && (best < 0 || freer(i, best))) best = i;",
@@ -70,6 +71,10 @@ MUTANTS = {
     "migration gate strict (F_d - F_s > theta)": ("< (int64_t)c.theta_num * dd * ds) break;",
                                                    "<= (int64_t)c.theta_num * dd * ds) break;"),
     "admission past a misfit head": ("if (need > in.free_blocks) break;", "if (need > in.free_blocks + need) break;"),
+    "headroom change applied one step late": ("c.headroom_change_step[next_change] <= st.steps",
+                                              "c.headroom_change_step[next_change] < st.steps"),
+    "headroom schedule ignored": ("for (int k = 0; k < c.num_tiers; ++k) H[k] = c.headroom_change_table[next_change * MAXK + k];",
+                                  "(void)0;"),
 }
 
 
@@ -79,7 +84,9 @@ def _pins_fail(so_path):
                   lambda: _closed_forms(so_path),
                   lambda: apins.check_tiny_drain_agreement(range(200), so_path=so_path),
                   lambda: _autoscale_closed_form(so_path),
-                  lambda: pins.check_threshold_equality(so_path=so_path)):
+                  lambda: pins.check_threshold_equality(so_path=so_path),
+                  lambda: adpins.check_tiny_schedule_agreement(range(150), so_path=so_path),
+                  lambda: adpins.check_dispatch_follows_the_change(so_path=so_path)):
         try:
             check()
         except AssertionError:
