@@ -252,6 +252,22 @@ int sim_reset(sim_t *sim);
  * allocated.  sim_run_static has no drain schedule. */
 int sim_set_drain(sim_t *sim, const uint32_t *drain_start_us, int on_device);
 
+/* Replaces the headroom tables (adaptive headroom, Sec. 6 "Adaptive
+ * headroom allocation": H_p adjusted while the system runs).
+ * headroom_blocks: host, [num_tables * max_tiers] in the layout of
+ * sim_tier_table_t.headroom_blocks (entries k >= the table's K are ignored),
+ * H_k >= 0 and M + sum_k H_k below 2^19 for every table, else SIM_ERR_ARG and
+ * nothing changes.  Every replica then uses its table's new values from the
+ * next step it processes (the next sim_run); each instance's headroom of the
+ * tiers present on it is recomputed.  The tables stay in force for later
+ * sim_reset and sim_load_trace calls.  Copied (the buffer may be reused
+ * when the call returns); queues a small kernel on the stream.  A replica
+ * stopped by a sim_run step limit has processed exactly that many steps, so
+ * a caller that changes the tables between calls of max_steps_per_replica E
+ * applies them at step indices E, 2E, ...: the same schedule runs the same
+ * way in every chunking. */
+int sim_set_headroom(sim_t *sim, const int32_t *headroom_blocks);
+
 /* Sets the order in which sim_run starts replicas: the persistent grid takes
  * replicas from a counter, and with an order set the k-th replica taken is
  * order[k].  Starting the replicas with the most work first shortens the

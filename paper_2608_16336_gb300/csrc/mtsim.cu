@@ -1593,6 +1593,29 @@ __global__ void k_init_state(Params p, const int *rep_table, const int *tbl_k, c
     }
 }
 
+// New headroom tables (adaptive headroom, sim_set_headroom): each replica's
+// H[k] from its table, and every instance's present-tier headroom sum
+// recomputed from its per-tier request counts (Sec. 3.3 Eq. 4: H_k once per
+// tier present).  One warp per replica.
+__global__ void k_set_headroom(Params p, const int *rep_table, const int *tbl_k, const int *tbl_h) {
+    const int lane = threadIdx.x & 31;
+    const int warps = (gridDim.x * blockDim.x) >> 5;
+    for (int r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < p.R; r += warps) {
+        unsigned char *b = p.blobs + (size_t)r * p.L.bytes;
+        const int tb = rep_table[r];
+        const int K = tbl_k[tb];
+        const int *hn = tbl_h + (size_t)tb * p.K;
+        for (int k = lane; k < p.K; k += 32) reinterpret_cast<int *>(b + p.L.h)[k] = k < K ? hn[k] : 0;
+        const uint16_t *cnt = reinterpret_cast<const uint16_t *>(b + p.L.cnt);
+        for (int i = lane; i < p.N; i += 32) {
+            int sum = 0;
+            for (int k = 0; k < K; ++k)
+                if (cnt[i * p.K + k] > 0) sum += hn[k];
+            reinterpret_cast<int *>(b + p.L.hr)[i] = sum;
+        }
+    }
+}
+
 __global__ void k_init_requests(sim_request_result_t *res, long long n) {
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x)
         reinterpret_cast<uint4 *>(res)[i] = make_uint4(0xFFFFFFFFu, kNone, kNone, 0u);
@@ -2248,6 +2271,35 @@ int sim_set_drain(sim_t *s, const uint32_t *drain_start_us, int on_device) {
                                     on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice, s->stream);
     if (e == cudaSuccess && !on_device) e = cudaStreamSynchronize(s->stream);  // the host buffer may be reused
     if (e != cudaSuccess) return cuda_fail(s, e, "sim_set_drain copy");
+    return SIM_OK;
+}
+
+int sim_set_headroom(sim_t *s, const int32_t *headroom_blocks) {
+    if (!s) return SIM_ERR_ARG;
+    if (!headroom_blocks) return fail(s, SIM_ERR_ARG, "headroom_blocks is NULL");
+    const int K = s->K;
+    for (int t = 0; t < s->ntables; ++t) {
+        long long sum = 0;
+        for (int k = 0; k < s->tbl_k[t]; ++k) {
+            const int h = headroom_blocks[(size_t)t * K + k];
+            if (h < 0) return fail(s, SIM_ERR_ARG, "table %d: negative headroom", t);
+            sum += h;
+        }
+        if (s->cl.blocks_per_instance + sum >= mt::kMaxKeyRange)
+            return fail(s, SIM_ERR_ARG, "table %d: M + sum of headroom must be below 2^19", t);
+    }
+    for (int t = 0; t < s->ntables; ++t)
+        for (int k = 0; k < K; ++k)
+            s->tbl_h[(size_t)t * K + k] = k < s->tbl_k[t] ? headroom_blocks[(size_t)t * K + k] : 0;
+    cudaError_t e = cudaMemcpyAsync(s->d_tbl_h, s->tbl_h.data(), s->tbl_h.size() * 4, cudaMemcpyHostToDevice, s->stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s->stream);  // the host vector may change at the next call
+    if (e != cudaSuccess) return cuda_fail(s, e, "sim_set_headroom copy");
+    if (s->loaded) {
+        mt::Params p = make_params(s, 0);
+        const int R = s->cl.num_replicas;
+        mt::k_set_headroom<<<(R + 7) / 8, 256, 0, s->stream>>>(p, s->d_rep_table, s->d_tbl_k, s->d_tbl_h);
+        return check_launch(s, "k_set_headroom");
+    }
     return SIM_OK;
 }
 

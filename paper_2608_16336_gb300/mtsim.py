@@ -81,7 +81,7 @@ class sim_allocator_t(ctypes.Structure):
 
 EXPORTS = ["sim_create", "sim_load_trace", "sim_reset", "sim_run", "sim_metrics", "sim_destroy",
            "sim_last_error", "sim_strerror", "sim_device_bytes", "sim_run_static", "sim_set_drain",
-           "sim_latency_stats", "sim_launch_info", "sim_set_order"]
+           "sim_latency_stats", "sim_launch_info", "sim_set_order", "sim_set_headroom"]
 SIM_STATIC_SCRATCH_BYTES = 32 << 20
 
 _LIB = None
@@ -121,6 +121,8 @@ def lib() -> ctypes.CDLL:
         L.sim_strerror.restype = ctypes.c_char_p
         L.sim_device_bytes.argtypes = [vp]
         L.sim_device_bytes.restype = ctypes.c_size_t
+        L.sim_set_headroom.argtypes = [vp, vp]
+        L.sim_set_headroom.restype = ctypes.c_int
         L.sim_set_order.argtypes = [vp, vp]
         L.sim_set_order.restype = ctypes.c_int
         L.sim_launch_info.argtypes = [vp, ctypes.POINTER(sim_launch_info_t)]
@@ -197,6 +199,10 @@ def sim_destroy(handle) -> None:
 
 def sim_device_bytes(handle) -> int:
     return int(lib().sim_device_bytes(handle))
+
+
+def sim_set_headroom(handle, headroom_ptr) -> int:
+    return _check(lib().sim_set_headroom(handle, headroom_ptr), handle)
 
 
 def sim_set_order(handle, order_ptr) -> int:
@@ -328,6 +334,14 @@ class Simulator:
         st = np.empty(self.w.num_replicas, STATS_DTYPE)
         sim_metrics(self.handle, None, st.ctypes.data, None, 0)
         return st
+
+    def set_headroom(self, tables) -> None:
+        """New headroom tables, [num_tables][max_tiers] (entries past a table's K ignored)."""
+        t = np.ascontiguousarray(tables, np.int32)
+        if t.shape != self._th.shape:
+            raise ValueError("tables must be [num_tables, max_tiers] = %s" % (self._th.shape,))
+        sim_set_headroom(self.handle, t.ctypes.data)
+        self._th = t
 
     def set_order(self, order) -> None:
         """Replica start order (a permutation of 0..R-1), or None for trace order."""
