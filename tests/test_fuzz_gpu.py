@@ -73,3 +73,48 @@ def test_random_clusters(chunk):
             parity.check_parity(w, event_log_capacity=1 << 14)
         except AssertionError as e:
             raise AssertionError("random case %d: %s" % (seed, e)) from e
+
+
+@pytest.mark.parametrize("chunk", range(4))
+def test_random_clusters_with_headroom_changes(chunk):
+    """The same random clusters run in random-size chunks of steps, with the
+    headroom table replaced at random between chunks (sim_set_headroom, the
+    adaptive-headroom mechanism); the oracle given the same schedule must
+    agree bit for bit."""
+    from oracle import oracle as O
+    from paper_2608_16336_gb300 import mtsim
+
+    total_changes = 0
+    for seed in range(chunk * 25, chunk * 25 + 25):
+        w = random_workload(1000 + seed)
+        if w.total_requests == 0:
+            continue
+        rng = np.random.default_rng(90_000 + seed)
+        k, m = w.tables_k[0], w.blocks_per_instance
+        steps = int(rng.integers(1, 400))
+        cap = 1 << 14
+        sched = []
+        sim = mtsim.Simulator(w, event_log_capacity=cap)
+        try:
+            sim.load()
+            j = 0
+            while sim.run(steps) > 0:
+                j += 1
+                if rng.random() < 0.7:
+                    tab = np.zeros_like(sim._th)
+                    tab[0, :k] = rng.integers(0, max(1, m // 2), size=k)
+                    sim.set_headroom(tab)
+                    sched.append((j * steps, [int(x) for x in tab[0, :k]]))
+            res, st, ev = sim.metrics()
+            events = [sim.events_of(ev, st, r) for r in range(w.num_replicas)]
+        finally:
+            sim.close()
+        total_changes += len(sched)
+        ref = O.run_workload(w, range(w.num_replicas), nthreads=8, log_capacity=cap,
+                             headroom_schedules={r: sched for r in range(w.num_replicas)})
+        try:
+            for r in range(w.num_replicas):
+                parity.compare_replica(w, r, res, st, events, ref[r])
+        except AssertionError as e:
+            raise AssertionError("random case %d (%d changes): %s" % (1000 + seed, len(sched), e)) from e
+    assert total_changes >= 25, total_changes  # the tables really changed mid-run
