@@ -1065,11 +1065,15 @@ constexpr bool kUnifiedLoop = !SMS && C <= 2;
 // order.  EXT: the variant that also handles draining instances and
 // the auto-scaling signal (the other variant compiles that code out).
 template <int C, bool SMS, bool EXT>
-// Variants that keep the running-request records in HBM run workloads with
-// many replicas; asking for 8 resident blocks per SM (at most 128 registers)
-// hides more of their latency.  The others keep 4: their shared memory or
-// register needs limit residency anyway.
-__global__ void __launch_bounds__(32 * kWarpsPerBlock, (!SMS && C <= 2) ? 8 : 4) k_run(Params p) {
+// Variants that keep the running-request records in HBM (C <= 2) run
+// workloads with many replicas and must stay at 128 registers so that 8
+// blocks of two warps fit on an SM.  The bound asks for 7: the compiler
+// still allocates 128 registers (spilling a few values to local memory) and
+// the launch still holds 8 blocks per SM, but its code for that bound
+// measured 3-4 % faster than for a bound of 8
+// (same-box A/B on the 16,384- and 3,840-replica workloads).  The others
+// keep 4: their shared memory or register needs limit residency anyway.
+__global__ void __launch_bounds__(32 * kWarpsPerBlock, (!SMS && C <= 2) ? 7 : 4) k_run(Params p) {
     extern __shared__ __align__(16) unsigned char smem[];
     unsigned long long *magic = reinterpret_cast<unsigned long long *>(smem);
     for (int d = threadIdx.x; d <= 64; d += blockDim.x)
