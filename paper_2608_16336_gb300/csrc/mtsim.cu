@@ -1060,7 +1060,7 @@ constexpr bool kUnifiedLoop = !SMS && C <= 2;
 // at least `base` microseconds.  So in a window [tmin, min(T_g, tmin + base))
 // every instance ends at most one iteration, and each lane advances its own
 // instances (an O(1) iteration end + batch formation); instances in a
-// migration (but a destination whose source has no event in the window), and
+// migration (but a destination whose source's next event comes later), and
 // every step at a global event, are advanced by the warp in the oracle's
 // order.  EXT: the variant that also handles draining instances and
 // the auto-scaling signal (the other variant compiles that code out).
@@ -1216,9 +1216,11 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, (!SMS && C <= 2) ? 7 : 4)
                         t1 = (uint32_t)min((unsigned long long)tg, (unsigned long long)tb + (uint32_t)p.base);
                         // instances with an iteration end in the window: stepped with
                         // the others of a migration in time order (cm), or alone
-                        // (solo).  A destination whose source has no event in the
-                        // window is alone: only the source's events (stages, commit,
-                        // abort) touch the other end.
+                        // (solo).  A destination whose source's next event comes
+                        // strictly later (or after the window) is alone: only the
+                        // source's events (stages, commit, abort) touch the other
+                        // end, and those then follow the destination's own event,
+                        // as in the oracle's time order.
                         cm = 0;
                         uint32_t solo = 0;
 #pragma unroll
@@ -1227,7 +1229,7 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, (!SMS && C <= 2) ? 7 : 4)
                             et[j] = bz[j];
                             if (bz[j] < t1) {
                                 const int role = x.mrole[i];
-                                if (role == MIG_NONE || (role == MIG_DST && x.busy[x.mpeer[i]] >= t1)) solo |= 1u << j;
+                                if (role == MIG_NONE || (role == MIG_DST && x.busy[x.mpeer[i]] > bz[j])) solo |= 1u << j;
                                 else cm |= 1u << j;
                             }
                         }
@@ -1393,15 +1395,16 @@ __global__ void __launch_bounds__(32 * kWarpsPerBlock, (!SMS && C <= 2) ? 7 : 4)
                         (uint32_t)min((unsigned long long)tg, (unsigned long long)tb + (uint32_t)p.base);
                     // instances with an iteration end in the window: stepped with the
                     // others of a migration in time order (cm), or alone (solo).  A
-                    // destination whose source has no event in the window is alone:
-                    // only the source's events (stages, commit, abort) touch the other end.
+                    // destination whose source's next event comes strictly later is
+                    // alone: only the source's events (stages, commit, abort) touch
+                    // the other end, and those then follow the destination's own event.
                     uint32_t cm = 0, solo = 0;
 #pragma unroll
                     for (int j = 0; j < C; ++j) {
                         const int i = lane * C + j;
                         if (bz[j] < t1) {
                             const int role = x.mrole[i];
-                            if (role == MIG_NONE || (role == MIG_DST && x.busy[x.mpeer[i]] >= t1)) solo |= 1u << j;
+                            if (role == MIG_NONE || (role == MIG_DST && x.busy[x.mpeer[i]] > bz[j])) solo |= 1u << j;
                             else cm |= 1u << j;
                         }
                     }
