@@ -309,3 +309,21 @@ def test_workload4_full_requests_sample():
     traces, bit-exact."""
     w = W.config(4, replicas=[0, 8191, 16383])
     parity.check_parity(w, event_log_capacity=1 << 14)
+
+
+def test_partitioned_runs_equal_the_whole():
+    """Replicas split into ranges by predicted work, as the multi-GPU
+    benchmark splits them across ranks, and simulated range by range give
+    the whole run's results bit for bit (replicas never interact)."""
+    reps = list(range(0, 3840, 32))  # 120 replicas of the sweep: every K, distribution and load
+    whole = W.config(2, replicas=reps, requests=800)
+    want = parity.run_gpu(whole, event_log_capacity=2048)
+    work = W.predicted_work(2, requests=800)[reps]
+    for lo, hi in W.partition(work, 3):
+        part = W.config(2, replicas=reps[lo:hi], requests=800)
+        got = parity.run_gpu(part, event_log_capacity=2048)
+        a, b = int(whole.offsets[lo]), int(whole.offsets[hi])
+        assert (got[0] == want[0][a:b]).all()
+        assert (got[1] == want[1][lo:hi]).all()
+        for r in range(hi - lo):
+            np.testing.assert_array_equal(got[2][r], want[2][lo + r])
