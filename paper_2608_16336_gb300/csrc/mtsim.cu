@@ -52,6 +52,7 @@
 
 #include <algorithm>
 #include <climits>
+#include <cstddef>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
@@ -95,10 +96,35 @@ enum : int { MIG_NONE = 0, MIG_SRC = 1, MIG_DST = 2 };
 // bucket's head is also kept in shared memory, so admission and the HoL demand
 // need no dependent HBM reads.
 
+// An instance's scalars, one record per instance: every field sits at a
+// fixed offset from the record, so the accesses to one instance share one
+// address.  13 words: lanes reading one field of consecutive instances hit
+// distinct shared-memory banks.
+struct InstRec {
+    uint32_t busy;                // end of the running iteration, or kNone when idle
+    int free_, resv, hol, hr;     // free KV blocks; reserved for inbound copies; HoL demand; present headroom
+    int key;                      // freeness key (dispatch, rebalancing)
+    uint32_t mreq;                // request being copied out (migration source)
+    int mcopied;                  // its blocks copied so far
+    uint32_t nf, minfin, drain;   // formations done; next finishing formation; drain start
+    uint16_t wmask;               // non-empty tier buckets
+    uint8_t nrun, pc, phase;      // running requests; iteration-ended flag; nf mod T
+    uint8_t mrole, mpeer, pad;    // migration role and peer
+};
+static_assert(sizeof(InstRec) == 52, "InstRec is 13 words");
+
+// x.busy[i] and the like: field F of instance i's record.
+template <typename T, int OFF>
+struct Field {
+    unsigned char *base;  // the replica's record array
+    __device__ __forceinline__ T &operator[](int i) const {
+        return *reinterpret_cast<T *>(base + i * (int)sizeof(InstRec) + OFF);
+    }
+};
+#define MT_FIELD(T, f) Field<T, (int)offsetof(InstRec, f)> f
+
 struct Layout {
-    uint32_t busy, free_, resv, hol, hr, key, mreq, mcopied, nf, minfin, drain;  // [N] x 4 B
-    uint32_t wmask;                                                      // [N] x 2 B
-    uint32_t nrun, pc, phase, mrole, mpeer;                               // [N] x 1 B
+    uint32_t inst;                                                       // [N] x InstRec
     uint32_t cnt;                                                        // [N*K] x 2 B
     uint32_t head, tail, hinfo;                                          // [N*K] x 4 B
     uint32_t h;                                                          // [K] x 4 B
@@ -148,10 +174,27 @@ struct Params {
 // memory, request state in HBM, slot records in either; scalars are warp-uniform
 // except t while lanes advance their own instances.
 struct Ctx {
-    uint32_t *busy, *mreq, *head, *tail, *hinfo, *nf, *minfin, *drain;
-    int *free_, *resv, *hol, *hr, *key, *mcopied, *h;
-    uint16_t *wmask, *cnt;
-    uint8_t *nrun, *pc, *phase, *mrole, *mpeer, *hist;
+    MT_FIELD(uint32_t, busy);
+    MT_FIELD(int, free_);
+    MT_FIELD(int, resv);
+    MT_FIELD(int, hol);
+    MT_FIELD(int, hr);
+    MT_FIELD(int, key);
+    MT_FIELD(uint32_t, mreq);
+    MT_FIELD(int, mcopied);
+    MT_FIELD(uint32_t, nf);
+    MT_FIELD(uint32_t, minfin);
+    MT_FIELD(uint32_t, drain);
+    MT_FIELD(uint16_t, wmask);
+    MT_FIELD(uint8_t, nrun);
+    MT_FIELD(uint8_t, pc);
+    MT_FIELD(uint8_t, phase);
+    MT_FIELD(uint8_t, mrole);
+    MT_FIELD(uint8_t, mpeer);
+    uint32_t *head, *tail, *hinfo;
+    int *h;
+    uint16_t *cnt;
+    uint8_t *hist;
     uint4 *mslot;                     // record of the request a migration source is copying out
     uint4 *slots;
     uint32_t *tset;                   // event-time set (C > 1)
@@ -960,23 +1003,10 @@ __device__ __forceinline__ void copy16(unsigned char *dst, const unsigned char *
 }
 
 __device__ __forceinline__ void bind_blob(Ctx &x, const Layout &L, unsigned char *blob) {
-    x.busy = reinterpret_cast<uint32_t *>(blob + L.busy);
-    x.free_ = reinterpret_cast<int *>(blob + L.free_);
-    x.resv = reinterpret_cast<int *>(blob + L.resv);
-    x.hol = reinterpret_cast<int *>(blob + L.hol);
-    x.hr = reinterpret_cast<int *>(blob + L.hr);
-    x.key = reinterpret_cast<int *>(blob + L.key);
-    x.mreq = reinterpret_cast<uint32_t *>(blob + L.mreq);
-    x.mcopied = reinterpret_cast<int *>(blob + L.mcopied);
-    x.nf = reinterpret_cast<uint32_t *>(blob + L.nf);
-    x.minfin = reinterpret_cast<uint32_t *>(blob + L.minfin);
-    x.drain = reinterpret_cast<uint32_t *>(blob + L.drain);
-    x.wmask = reinterpret_cast<uint16_t *>(blob + L.wmask);
-    x.nrun = blob + L.nrun;
-    x.pc = blob + L.pc;
-    x.phase = blob + L.phase;
-    x.mrole = blob + L.mrole;
-    x.mpeer = blob + L.mpeer;
+    unsigned char *ib = blob + L.inst;
+    x.busy.base = x.free_.base = x.resv.base = x.hol.base = x.hr.base = x.key.base = ib;
+    x.mreq.base = x.mcopied.base = x.nf.base = x.minfin.base = x.drain.base = ib;
+    x.wmask.base = x.nrun.base = x.pc.base = x.phase.base = x.mrole.base = x.mpeer.base = ib;
     x.cnt = reinterpret_cast<uint16_t *>(blob + L.cnt);
     x.head = reinterpret_cast<uint32_t *>(blob + L.head);
     x.tail = reinterpret_cast<uint32_t *>(blob + L.tail);
@@ -1068,11 +1098,11 @@ template <int C, bool SMS, bool EXT>
 // Variants that keep the running-request records in HBM (C <= 2) run
 // workloads with many replicas and must stay at 128 registers so that 8
 // blocks of two warps fit on an SM.  The bound asks for 7: the compiler
-// still allocates 128 registers (spilling a few values to local memory) and
-// the launch still holds 8 blocks per SM, but its code for that bound
-// measured 3-4 % faster than for a bound of 8
-// (same-box A/B on the 16,384- and 3,840-replica workloads).  The others
-// keep 4: their shared memory or register needs limit residency anyway.
+// still allocates 128 registers and the launch still holds 8 blocks per SM,
+// but its code for that bound measured faster than for a bound of 8 (1-4 %,
+// same-box A/B on the 16,384- and 3,840-replica workloads); a bound of 10
+// (96 registers, 9-10 blocks) was 10-16 % slower.  The others keep 4: their
+// shared memory or register needs limit residency anyway.
 __global__ void __launch_bounds__(32 * kWarpsPerBlock, (!SMS && C <= 2) ? 7 : 4) k_run(Params p) {
     extern __shared__ __align__(16) unsigned char smem[];
     unsigned long long *magic = reinterpret_cast<unsigned long long *>(smem);
@@ -1563,23 +1593,15 @@ __global__ void k_init_state(Params p, const int *rep_table, const int *tbl_k, c
         const int tb = rep_table[r];
         const int K = tbl_k[tb];
         for (int i = lane; i < N; i += 32) {
-            reinterpret_cast<uint32_t *>(b + L.busy)[i] = kNone;
-            reinterpret_cast<int *>(b + L.free_)[i] = p.M;
-            reinterpret_cast<int *>(b + L.resv)[i] = 0;
-            reinterpret_cast<int *>(b + L.hol)[i] = 0;
-            reinterpret_cast<int *>(b + L.hr)[i] = 0;
-            reinterpret_cast<int *>(b + L.key)[i] = 0;
-            reinterpret_cast<uint32_t *>(b + L.mreq)[i] = kNone;
-            reinterpret_cast<int *>(b + L.mcopied)[i] = 0;
-            reinterpret_cast<uint32_t *>(b + L.nf)[i] = 0;
-            reinterpret_cast<uint32_t *>(b + L.minfin)[i] = kNone;
-            reinterpret_cast<uint32_t *>(b + L.drain)[i] = p.drain_src ? p.drain_src[(size_t)r * N + i] : kNone;
-            reinterpret_cast<uint16_t *>(b + L.wmask)[i] = 0;
-            b[L.nrun + i] = 0;
-            b[L.pc + i] = 0;
-            b[L.phase + i] = 0;
-            b[L.mrole + i] = MIG_NONE;
-            b[L.mpeer + i] = 0;
+            InstRec v;
+            memset(&v, 0, sizeof v);
+            v.busy = kNone;
+            v.free_ = p.M;
+            v.mreq = kNone;
+            v.minfin = kNone;
+            v.drain = p.drain_src ? p.drain_src[(size_t)r * N + i] : kNone;
+            v.mrole = MIG_NONE;
+            reinterpret_cast<InstRec *>(b + L.inst)[i] = v;
         }
         for (int q = lane; q < N * p.TH; q += 32) b[L.hist + q] = 0;
         for (int i = lane; i < NK; i += 32) {
@@ -1618,7 +1640,7 @@ __global__ void k_set_headroom(Params p, const int *rep_table, const int *tbl_k,
             int sum = 0;
             for (int k = 0; k < K; ++k)
                 if (cnt[i * p.K + k] > 0) sum += hn[k];
-            reinterpret_cast<int *>(b + p.L.hr)[i] = sum;
+            reinterpret_cast<InstRec *>(b + p.L.inst)[i].hr = sum;
         }
     }
 }
@@ -1732,28 +1754,12 @@ inline Layout make_layout(int N, int K, int T) {
         o += bytes;
         return at;
     };
-    L.busy = take(4u * N, 16);
-    L.free_ = take(4u * N, 16);
-    L.resv = take(4u * N, 16);
-    L.hol = take(4u * N, 16);
-    L.hr = take(4u * N, 16);
-    L.key = take(4u * N, 16);
-    L.mreq = take(4u * N, 16);
-    L.mcopied = take(4u * N, 16);
-    L.nf = take(4u * N, 16);
-    L.minfin = take(4u * N, 16);
-    L.drain = take(4u * N, 16);
+    L.inst = take((uint32_t)sizeof(InstRec) * N, 16);
     L.head = take(4u * N * K, 16);
     L.tail = take(4u * N * K, 16);
     L.hinfo = take(4u * N * K, 16);
     L.h = take(4u * K, 16);
-    L.wmask = take(2u * N, 16);
     L.cnt = take(2u * N * K, 16);
-    L.nrun = take(N, 16);
-    L.pc = take(N, 16);
-    L.phase = take(N, 16);
-    L.mrole = take(N, 16);
-    L.mpeer = take(N, 16);
     L.hist = take((uint32_t)N * hist_stride(T), 16);
     L.mslot = take(16u * N, 16);
     L.bytes = (o + 15u) & ~15u;
