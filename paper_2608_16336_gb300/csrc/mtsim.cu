@@ -1743,7 +1743,12 @@ struct Launch {
 
 inline int lanes_c(int N) { return N <= 32 ? 1 : N <= 64 ? 2 : N <= 128 ? 4 : 8; }
 
-inline int hist_stride(int T) { return (T + 3) & ~3; }
+// Bytes per instance of the growth histogram: T rounded up to an odd number
+// of words, so lanes reading one entry of consecutive instances hit distinct
+// banks (1,024-replica workload +0.8 %; the same odd stride for the bucket
+// arrays, as one {head, tail, info, count} record per tier, was 3 % slower
+// on the 16,384-replica workload).
+inline int hist_stride(int T) { return (((T + 3) >> 2) | 1) << 2; }
 
 inline Layout make_layout(int N, int K, int T) {
     Layout L;
