@@ -422,7 +422,8 @@ def bench_other(torch, mtsim, workloads, cid: int, stream, args) -> dict:
 
 def time_latency_stats(torch, mtsim, sim, w, stream, reps: int = 10) -> dict:
     """CUDA-event time of the per-tier latency reduction (sim_latency_stats) over the
-    finished simulation, device output, outside the timed step.  Its inputs
+    finished simulation, device output, outside the timed step: the histogram
+    pass, the percentile buckets and the exact selection passes.  Its inputs
     (16 + 4 + 2 + 1 bytes per request) are larger than L2 at this size."""
     R, Q = w.num_replicas, w.total_requests
     kmax = max(w.tables_k)
@@ -440,8 +441,10 @@ def time_latency_stats(torch, mtsim, sim, w, stream, reps: int = 10) -> dict:
     nbytes = Q * (16 + 4 + 2 + 1) + out.numel()
     peak, kind = measured_peak_hbm()
     gbs = nbytes / (ms / 1e3) / 1e9
-    return {"kernel": "k_latency_hist + k_latency_pct (sim_latency_stats, output clear included)",
-            "work": "per-tier TTFT/TBT/E2E histograms and percentiles of every request",
+    return {"kernel": "sim_latency_stats: k_latency_hist, k_latency_pct and up to four k_latency_refine + "
+                      "k_latency_step selection passes (output clear included)",
+            "work": "per-tier TTFT/TBT/E2E histograms and exact nearest-rank P50/P90/P99 of every request; "
+                    "algorithmic bytes = one read of the inputs, which each selection pass still open reads again",
             "bound": "hbm", "ms": ms, "algorithmic_bytes_per_launch": nbytes, "achieved": gbs, "peak": peak,
             "peak_kind": kind, "unit": "GB/s", "frac": gbs / peak}
 
