@@ -73,6 +73,14 @@ MUTANTS = {
     "admission past a misfit head": ("if (need > in.free_blocks) break;", "if (need > in.free_blocks + need) break;"),
     "headroom change applied one step late": ("c.headroom_change_step[next_change] <= st.steps",
                                               "c.headroom_change_step[next_change] < st.steps"),
+    "running candidate of the highest priority": ("if (a.tier != b.tier ? a.tier > b.tier :",
+                                                  "if (a.tier != b.tier ? a.tier < b.tier :"),
+    "queued candidate from the highest-priority bucket": (
+        "for (int k = c.num_tiers - 1; k >= 0; --k)\n                if (!S.waiting[k].empty()) { kq = k; break; }",
+        "for (int k = 0; k < c.num_tiers; ++k)\n                if (!S.waiting[k].empty()) { kq = k; break; }"),
+    "aborted copy keeps the destination's blocks": (
+        "d.free_blocks += s.mig_copied;   /* copied blocks are released on the destination */",
+        "/* copied blocks are kept */"),
     "headroom schedule ignored": ("for (int k = 0; k < c.num_tiers; ++k) H[k] = c.headroom_change_table[next_change * MAXK + k];",
                                   "(void)0;"),
 }
